@@ -77,6 +77,8 @@ def _load():
             "oracle_dequant_fp8": (None, [_p, _p, ctypes.c_int, _i64, _i64, _p,
                                           _i64, _p]),
             "oracle_gemm_f64": (None, [_p, _p, _i64, _i64, _i64, _p, _p, _p]),
+            "oracle_round_bf16": (ctypes.c_uint16, [ctypes.c_double]),
+            "oracle_round_bf16_array": (None, [_p, _i64, _p]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -128,6 +130,18 @@ def e4m3_encode(v: float) -> int:
 
 def bf16_to_f32(bits: int) -> float:
     return _load().oracle_bf16_to_f32(int(bits))
+
+
+def round_bf16(v: float) -> int:
+    """bf16 bits of the nearest bf16 to an fp64 value (ties to even)."""
+    return _load().oracle_round_bf16(float(v))
+
+
+def round_bf16_array(v: np.ndarray) -> np.ndarray:
+    v = np.ascontiguousarray(v, np.float64)
+    out = np.empty(v.shape, np.uint16)
+    _load().oracle_round_bf16_array(_ptr(v), v.size, _ptr(out))
+    return out
 
 
 # ---------------------------------------------------------------- scales ---

@@ -77,6 +77,25 @@ float oracle_bf16_to_f32(uint16_t b) {
   return f;
 }
 
+/* Nearest bf16 (8-bit significand, binary32 exponent range) to an fp64
+ * value, ties to even; used to state the expected bf16 output of the linear
+ * (the layer writes bf16).  Finite inputs; overflow gives +-inf. */
+uint16_t oracle_round_bf16(double v) {
+  uint16_t sign = signbit(v) ? 0x8000 : 0;
+  double a = fabs(v);
+  if (a == 0.0) return sign;
+  int e2;
+  frexp(a, &e2);               /* a in [2^(e2-1), 2^e2) */
+  int E = e2 - 1;
+  if (E < -126) E = -126;      /* subnormal range: fixed step 2^-133 */
+  double q = round_half_even(ldexp(a, 7 - E));   /* significand in units of 2^(E-7) */
+  if (q >= 256.0) { q /= 2.0; E += 1; }          /* carried into the next binade */
+  if (E > 127) return sign | 0x7F80;
+  uint32_t mant = (uint32_t)q;                   /* 128..255 normal, < 128 subnormal */
+  uint32_t bits = (mant >= 128) ? ((uint32_t)(E + 127) << 7) | (mant - 128) : mant;
+  return sign | (uint16_t)bits;
+}
+
 /* ------------------------------------------------------------------ */
 /* e2m1 (FP4) -- the element type of NVFP4 (NVIDIA 2025, cited in Sec. 4)  */
 /* code bits: s | e1 e0 | m, exponent bias 1, no inf/NaN.              */
@@ -340,4 +359,9 @@ void oracle_gemm_f64(const double *a, const double *w, int64_t M, int64_t N,
       for (int64_t k = 0; k < K; ++k) s += w[n * K + k] * w[n * K + k];
       norm_w[n] = sqrt(s);
     }
+}
+
+void oracle_round_bf16_array(const double *v, int64_t n, uint16_t *out) {
+#pragma omp parallel for schedule(static)
+  for (int64_t i = 0; i < n; ++i) out[i] = oracle_round_bf16(v[i]);
 }

@@ -1,0 +1,53 @@
+// Internal declarations shared by the translation units of libqlin.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <algorithm>
+
+#include "qlin.h"
+#include "qlin_device.cuh"
+
+namespace qlin {
+
+// ---- quantizers (qlin_quant.cu) ----
+cudaError_t launch_amax(const void* x, int64_t n_elems, unsigned* amax_bits, cudaStream_t s,
+                        int num_sms);
+cudaError_t launch_quant_nvfp4(const void* x, int64_t M, int64_t K, const float* scale_src,
+                               bool dynamic, const qlin_nvfp4_t& out, cudaStream_t s,
+                               int num_sms);
+cudaError_t launch_quant_fp8(const void* x, int64_t M, int64_t K, const float* scale_src,
+                             bool dynamic, const qlin_fp8_t& out, cudaStream_t s, int num_sms);
+cudaError_t launch_quant_fp8_rows(const void* w, int64_t N, int64_t K, const qlin_fp8_t& out,
+                                  cudaStream_t s, int num_sms);
+
+// ---- GEMMs (qlin_gemm.cu) ----
+struct GemmArgs {
+  bool fp4;                 // NVFP4 (true) or FP8
+  const void* a_codes;      // [M, K/2] or [M, K] bytes
+  const void* w_codes;      // [N, K/2] or [N, K] bytes
+  const uint8_t* sfa;       // swizzled block scales (NVFP4)
+  const uint8_t* sfb;
+  const float* sdec_a;      // tensor scale of A
+  const float* sdec_w;      // tensor scale of W (NVFP4) / per-channel or single (FP8)
+  int w_per_channel;        // FP8: 1 if sdec_w has N entries
+  void* y;                  // bf16 [M, N] or null
+  int64_t M, N, K;
+  // fused NVFP4 re-quantization of y's columns [rq_col0, rq_col0 + rq_cols)
+  const float* next_scale;  // null = off
+  uint8_t* rq_codes;
+  uint8_t* rq_scales;
+  float* rq_tensor_scale;
+  int64_t rq_col0, rq_cols;
+};
+cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned* err,
+                        uint64_t timeout_ns);
+cudaError_t launch_wait_selftest(uint64_t timeout_ns, cudaStream_t s, unsigned* err);
+
+// Resolves cuTensorMapEncodeTiled through the runtime (no libcuda link).
+CUresult encode_tensor_map_2d_u8(CUtensorMap* map, const void* base, uint64_t inner_bytes,
+                                 uint64_t rows, uint32_t box_inner, uint32_t box_rows);
+
+}  // namespace qlin

@@ -112,11 +112,13 @@ def nvfp4_mlp_up(M=M_TOKENS, K=HIDDEN, N=MLP, seed=2):
 
 
 def translator(M=512, seed=3):
-    """Translator-shaped small-M linears: x [512,1024], W1 [2560,1024],
-    W2 [1024,2560], sigma 0.03."""
-    x = act_normal(seed, M, 1024)
+    """Translator-shaped small-M linears (batch 1, 512 tokens): x1 [512, 1024]
+    feeds W1 [2560, 1024]; x2 [512, 2560] feeds W2 [1024, 2560]; activations
+    N(0, 1) (x2 from default_rng([seed, 2])), weights N(0, 0.03^2)."""
+    x1 = act_normal(seed, M, 1024)
+    x2 = bf16_bits(_normal(np.random.default_rng([seed, 2]), (M, 2560)))
     w1, w2 = weights(seed, [(2560, 1024), (1024, 2560)], 0.03)
-    return x, w1, w2
+    return x1, x2, w1, w2
 
 
 STACK_LAYERS = (("qkv", 3 * HIDDEN, HIDDEN), ("out", HIDDEN, HIDDEN),

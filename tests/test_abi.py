@@ -1,0 +1,89 @@
+"""The C-ABI library loads, exports every function include/qlin.h declares,
+and rejects bad arguments on the host before any CUDA call (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from conftest import ROOT
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_21849_gb300 import build, qlin
+    build.build()
+    return qlin.load_library()
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "qlin.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(qlin_\w+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ("qlin_quantize_weight", "qlin_quantize_act_nvfp4", "qlin_quantize_act_fp8",
+              "qlin_gemm_nvfp4", "qlin_gemm_fp8", "qlin_linear_fused"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    from paper_2609_21849_gb300 import qlin
+    for name in _declared():
+        assert hasattr(lib, name), name
+    assert sorted(qlin.EXPORTS) == _declared()
+
+
+def test_scale_bytes_and_workspace(lib):
+    from paper_2609_21849_gb300 import qlin
+    assert qlin.qlin_nvfp4_scale_bytes(128, 256) == 2048
+    assert qlin.qlin_nvfp4_scale_bytes(129, 256) == 4096
+    assert qlin.qlin_nvfp4_scale_bytes(4608, 3072) == 36 * 48 * 512
+    assert qlin.qlin_nvfp4_scale_bytes(128, 100) == 0
+    assert qlin.qlin_workspace_size(1, 64) >= 4
+
+
+def test_argument_errors_return_before_launch(lib):
+    from paper_2609_21849_gb300 import qlin
+    d = qlin.NVFP4Desc(16, 16, 16, 128, 256)  # fake, never dereferenced
+    # null input
+    assert lib.qlin_quantize_act_nvfp4(None, 128, 256, None, ctypes.byref(d), 16, 256, None) == 1
+    # K not a multiple of 64
+    d2 = qlin.NVFP4Desc(16, 16, 16, 128, 96)
+    assert lib.qlin_quantize_act_nvfp4(16, 128, 96, None, ctypes.byref(d2), 16, 256, None) == 1
+    # rows mismatch between the descriptor and the call
+    assert lib.qlin_quantize_act_nvfp4(16, 64, 256, None, ctypes.byref(d), 16, 256, None) == 1
+    # misaligned input pointer
+    assert lib.qlin_quantize_act_nvfp4(24, 128, 256, None, ctypes.byref(d), 16, 256, None) == 3
+    # dynamic scale without workspace
+    assert lib.qlin_quantize_act_nvfp4(16, 128, 256, None, ctypes.byref(d), None, 0, None) == 6
+    # GEMM: K mismatch, N not a multiple of 64, nothing to write
+    a = qlin.NVFP4Desc(16, 16, 16, 128, 256)
+    w = qlin.NVFP4Desc(16, 16, 16, 256, 512)
+    assert lib.qlin_gemm_nvfp4(ctypes.byref(a), ctypes.byref(w), 16, None) == 1
+    w = qlin.NVFP4Desc(16, 16, 16, 96, 256)
+    assert lib.qlin_gemm_nvfp4(ctypes.byref(a), ctypes.byref(w), 16, None) == 1
+    w = qlin.NVFP4Desc(16, 16, 16, 256, 256)
+    assert lib.qlin_linear_fused(ctypes.byref(a), ctypes.byref(w), None, None, None, 0, None) == 1
+    # re-quantization window outside the output
+    q = qlin.NVFP4Desc(16, 16, 16, 128, 128)
+    assert lib.qlin_linear_fused(ctypes.byref(a), ctypes.byref(w), 16, 16, ctypes.byref(q), 192,
+                                 None) == 1
+    # FP8: per-channel activation descriptor is rejected; unknown weight format
+    f = qlin.FP8Desc(16, 16, 128, 256, 1)
+    assert lib.qlin_quantize_act_fp8(16, 128, 256, 16, ctypes.byref(f), None, 0, None) == 1
+    assert lib.qlin_quantize_weight(16, 128, 256, 7, ctypes.byref(f), None, 0, None) == 2
+    assert lib.qlin_status_str(5) == b"device wait timed out"
+
+
+def test_python_binding_fails_loudly_without_library(tmp_path):
+    from paper_2609_21849_gb300 import qlin
+    saved = qlin._lib
+    try:
+        qlin._lib = None
+        with pytest.raises(RuntimeError, match="not built"):
+            qlin.load_library(str(tmp_path / "missing.so"))
+    finally:
+        qlin._lib = saved

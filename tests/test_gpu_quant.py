@@ -1,0 +1,128 @@
+"""GPU parity of the quantizers (Sec. 4, "Quantization": run-time FP8 / NVFP4
+activation quantization and offline weight quantization): codes, block scales
+and tensor scales must equal the CPU oracle's bit for bit."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import oracle
+from paper_2609_21849_gb300 import qlin, synthetic
+
+from conftest import read_golden
+
+pytestmark = pytest.mark.gpu
+
+if torch.cuda.is_available():
+    from gpu_util import assert_nvfp4_equal, f32, nvfp4_to_host, to_dev, u8
+
+
+RAGGED = [(1, 64), (3, 128), (130, 192), (257, 320), (128, 4096), (333, 1088)]
+
+
+@pytest.mark.parametrize("M,K", RAGGED)
+@pytest.mark.parametrize("dynamic", [True, False])
+def test_nvfp4_act_ragged(M, K, dynamic):
+    x = synthetic.act_entry_outliers(M * 7 + K, M, K)
+    s_dec = None if dynamic else 0.0123
+    ref = oracle.quant_nvfp4(x, s_dec)
+    static = None if dynamic else torch.tensor([np.float32(s_dec)], device="cuda")
+    q = qlin.qlin_quantize_act_nvfp4(to_dev(x), static_scale=static)
+    assert qlin.qlin_sync_status() == 0
+    assert_nvfp4_equal(q, ref, f"[{M},{K}] dynamic={dynamic}")
+
+
+def test_nvfp4_tiny_workload():
+    x, w = synthetic.tiny_nvfp4()
+    q = qlin.qlin_quantize_act_nvfp4(to_dev(x))
+    assert_nvfp4_equal(q, oracle.quant_nvfp4(x), "tiny x")
+    qw = qlin.qlin_quantize_weight(to_dev(w), qlin.QLIN_FMT_NVFP4)
+    assert_nvfp4_equal(qw, oracle.quant_nvfp4(w), "tiny W")
+
+
+def test_nvfp4_act_full_size_mlp_up():
+    # the 4608 x 3072 activation of the MLP up-projection, full tensor
+    x = synthetic.act_entry_outliers(2, synthetic.M_TOKENS, synthetic.HIDDEN)
+    ref = oracle.quant_nvfp4(x)
+    q = qlin.qlin_quantize_act_nvfp4(to_dev(x))
+    assert qlin.qlin_sync_status() == 0
+    assert_nvfp4_equal(q, ref, "4608x3072 dynamic")
+    # static mode with the calibrated scale gives the same result
+    q2 = qlin.qlin_quantize_act_nvfp4(to_dev(x), static_scale=q.tensor_scale.clone())
+    assert_nvfp4_equal(q2, ref, "4608x3072 static")
+
+
+def test_nvfp4_weight_full_size():
+    (w,) = synthetic.weights(2, [(synthetic.MLP, synthetic.HIDDEN)], 0.02)
+    q = qlin.qlin_quantize_weight(to_dev(w), qlin.QLIN_FMT_NVFP4)
+    assert_nvfp4_equal(q, oracle.quant_nvfp4(w), "W 12288x3072")
+
+
+def test_nvfp4_hand_worked_blocks_on_gpu():
+    # every golden block, placed in different rows / block positions
+    lines = read_golden("nvfp4_blocks.txt")
+    blocks = []
+    for i in range(0, len(lines), 4):
+        if float(lines[i].split()[3]) == 1.0:
+            blocks.append([float(v) for v in lines[i + 1].split()[1:]])
+    K = 64 * 2
+    x = np.zeros((len(blocks) * 3, K), np.float32)
+    for r in range(x.shape[0]):
+        for b in range(K // 16):
+            x[r, b * 16:(b + 1) * 16] = blocks[(r + b) % len(blocks)]
+    bits = synthetic.bf16_bits(x)
+    ref = oracle.quant_nvfp4(bits, 1.0)
+    q = qlin.qlin_quantize_act_nvfp4(to_dev(bits), static_scale=torch.ones(1, device="cuda"))
+    assert_nvfp4_equal(q, ref, "golden blocks")
+
+
+def test_nvfp4_extreme_values():
+    # zeros, signed zeros, subnormal bf16, huge values, and an all-zero tensor
+    rng = np.random.default_rng(0)
+    K = 256
+    x = (rng.standard_normal((64, K)) * 10.0 ** rng.integers(-38, 38, (64, K))).astype(np.float32)
+    x[0] = 0.0
+    x[1] = -0.0
+    x[2, ::3] = 1e-40
+    x[3, :16] = 3e38
+    bits = synthetic.bf16_bits(np.clip(np.nan_to_num(x, posinf=3e38, neginf=-3e38), -3e38, 3e38))
+    for s in (None, 1.0, 1e-30, 1e30):
+        ref = oracle.quant_nvfp4(bits, s)
+        st = None if s is None else torch.tensor([np.float32(s)], device="cuda")
+        q = qlin.qlin_quantize_act_nvfp4(to_dev(bits), static_scale=st)
+        assert_nvfp4_equal(q, ref, f"extreme s={s}")
+    z = np.zeros((5, 64), np.uint16)
+    q = qlin.qlin_quantize_act_nvfp4(to_dev(z))
+    assert_nvfp4_equal(q, oracle.quant_nvfp4(z), "all zero")
+
+
+@pytest.mark.parametrize("M,K", RAGGED)
+@pytest.mark.parametrize("dynamic", [True, False])
+def test_fp8_act_ragged(M, K, dynamic):
+    x = synthetic.act_channel_gain(M + K, M, K)
+    s_dec = None if dynamic else 0.37
+    rc, rs = oracle.quant_fp8(x, s_dec)
+    static = None if dynamic else torch.tensor([np.float32(s_dec)], device="cuda")
+    q = qlin.qlin_quantize_act_fp8(to_dev(x), static_scale=static)
+    assert qlin.qlin_sync_status() == 0
+    assert f32(q.scale)[0].view(np.uint32) == np.float32(rs).view(np.uint32)
+    assert np.array_equal(u8(q.codes), rc)
+
+
+def test_fp8_act_full_size():
+    x = synthetic.act_channel_gain(1, synthetic.M_TOKENS, synthetic.HIDDEN)
+    rc, rs = oracle.quant_fp8(x)
+    q = qlin.qlin_quantize_act_fp8(to_dev(x))
+    assert f32(q.scale)[0] == rs
+    assert np.array_equal(u8(q.codes), rc)
+
+
+@pytest.mark.parametrize("N,K", [(1, 64), (65, 192), (3072, 3072)])
+def test_fp8_weight_per_channel(N, K):
+    (w,) = synthetic.weights(N, [(N, K)], 0.02)
+    w = w.copy()
+    w[0] = 0  # an all-zero channel takes scale 1
+    rc, rs = oracle.quant_fp8_rows(w)
+    q = qlin.qlin_quantize_weight(to_dev(w), qlin.QLIN_FMT_FP8)
+    assert np.array_equal(f32(q.scale).view(np.uint32), rs.view(np.uint32))
+    assert np.array_equal(u8(q.codes), rc)

@@ -117,3 +117,23 @@ def test_bf16_widening(oracle):
     for bits, val in [(0x3F80, 1.0), (0xC000, -2.0), (0x0000, 0.0), (0x7F7F, 3.3895313892515355e38),
                       (0x0001, 9.183549615799121e-41)]:
         assert oracle.bf16_to_f32(bits) == np.float32(val)
+
+
+def test_round_bf16_matches_fp32_rounding(oracle):
+    # On fp32-representable values the direct fp64 -> bf16 rounding must agree
+    # with the generator's independent fp32 -> bf16 rounding.
+    from paper_2609_21849_gb300 import synthetic
+    rng = np.random.default_rng(5)
+    v = np.concatenate([rng.standard_normal(4000) * 10.0 ** rng.integers(-30, 30, 4000),
+                        [1e-40, -3e-39, 0.0, -0.0]]).astype(np.float32)
+    got = oracle.round_bf16_array(v.astype(np.float64))
+    assert np.array_equal(got, synthetic.bf16_bits(v))
+
+
+def test_round_bf16_ties_and_single_rounding(oracle):
+    assert oracle.round_bf16(1.0 + 2.0 ** -8) == 0x3F80            # tie -> even
+    assert oracle.round_bf16(1.0 + 3 * 2.0 ** -8) == 0x3F82        # tie -> even (up)
+    # just above a tie: a double rounding through fp32 would land on the tie
+    # and go to even; rounding once from fp64 goes up
+    assert oracle.round_bf16(1.0 + 2.0 ** -8 + 2.0 ** -40) == 0x3F81
+    assert oracle.round_bf16(-2.0) == 0xC000
