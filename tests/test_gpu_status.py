@@ -27,7 +27,7 @@ def test_bounded_wait_expires_and_reports_timeout():
 
 
 def test_misaligned_device_pointers_are_rejected():
-    buf = torch.zeros(4096, dtype=torch.uint8, device="cuda")
+    buf = torch.zeros(128 * 64 * 2 + 64, dtype=torch.uint8, device="cuda")
     x = buf[2:2 + 128 * 64 * 2].view(torch.bfloat16).view(128, 64)  # 2-byte offset
     with pytest.raises(qlin.QlinError) as e:
         qlin.qlin_quantize_act_nvfp4(x)
