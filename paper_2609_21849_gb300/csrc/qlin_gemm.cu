@@ -20,6 +20,7 @@
 //               thread-local).
 // Tiles are 128 x BN output blocks, scheduled m-fastest so consecutive CTAs
 // share a weight tile in L2.  Every wait is bounded (see WaitCtl).
+#include <cstring>
 #include <mutex>
 
 #include "qlin_internal.h"
@@ -32,7 +33,8 @@ constexpr int kBM = 128;
 constexpr int kRowBytes = 128;      // bytes of K per stage and row: one swizzle row
 constexpr int kStepsPerStage = 4;   // one MMA per 32 bytes of K
 constexpr int kEpiWarps = 8;
-constexpr int kThreads = (2 + kEpiWarps) * 32;
+constexpr int kEpiWarp0 = 3;                      // warps 0-2: producer, MMA, scale copies
+constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
 constexpr int kSmemBudget = 232448 - 2048;  // opt-in shared memory minus barriers/alignment
 
 constexpr int pow2_at_least(int x) {
@@ -49,15 +51,17 @@ struct Cfg {
   static constexpr int kSfaBytes = kFp4 ? kStepsPerStage * 512 : 0;
   static constexpr int kSfbBytes = kFp4 ? kSfbAtoms * kStepsPerStage * 512 : 0;
   static constexpr int kStageBytes = kABytes + kBBytes + kSfaBytes + kSfbBytes;
-  static constexpr int kStagesRaw = kSmemBudget / kStageBytes;
+  // epilogue staging: per epilogue warp two 32 x 32 bf16 boxes (2 KB each)
+  static constexpr int kOutBytes = kEpiWarps * 2 * 2048;
+  static constexpr int kStagesRaw = (kSmemBudget - kOutBytes) / kStageBytes;
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
   static constexpr int kNumAcc = (kFp4 && kBN == 256) ? 1 : 2;
   static constexpr int kSfColsPerStep = kFp4 ? 4 + 4 * kSfbAtoms : 0;
   static constexpr int kSfColBase = kNumAcc * kBN;
   static constexpr int kTmemCols =
       pow2_at_least(kSfColBase + kStages * kStepsPerStage * kSfColsPerStep);
-  static constexpr int kBarrierBytes = 256;
-  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarrierBytes;
+  static constexpr int kBarrierBytes = 512;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kOutBytes + kBarrierBytes;
   static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
   static_assert(kTmemCols <= 512, "TMEM budget");
   static_assert(kSmemBytes <= 232448, "shared memory budget");
@@ -102,35 +106,47 @@ __device__ __forceinline__ void st_global_v4(void* p, uint32_t a, uint32_t b, ui
                : "memory");
 }
 
-template <bool kFp4, int kBN, bool kRequant>
+template <bool kFp4, int kBN, int kCM, bool kRequant>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_a,
-                const __grid_constant__ CUtensorMap tmap_b, const KParams p) {
+                const __grid_constant__ CUtensorMap tmap_b,
+                const __grid_constant__ CUtensorMap tmap_y, const KParams p) {
   using C = Cfg<kFp4, kBN>;
+  // kCM CTAs of a cluster take kCM consecutive M tiles of the same N tile;
+  // each loads 1/kCM of the weight tile (and of its scales) and multicasts
+  // it to all, so W is read from L2 once per cluster.
+  constexpr int kBRows = kBN / kCM;
+  constexpr uint16_t kMask = (uint16_t)((1u << kCM) - 1u);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
+  uint8_t* out_stage = smem + C::kStages * C::kStageBytes;   // epilogue staging boxes
+  uint64_t* full = reinterpret_cast<uint64_t*>(out_stage + C::kOutBytes);
   uint64_t* empty = full + C::kStages;
-  uint64_t* tmem_full = empty + C::kStages;
+  uint64_t* sf_ready = empty + C::kStages;   // NVFP4: the stage's scales are in TMEM
+  uint64_t* tmem_full = sf_ready + C::kStages;
   uint64_t* tmem_empty = tmem_full + 2;
   uint64_t* mma_done = tmem_empty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  uint64_t* sf_done = mma_done + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sf_done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const int rank = kCM > 1 ? (int)cluster_ctarank() : 0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], kCM);   // one arrival from the MMA warp of each CTA
+      mbar_init(&sf_ready[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tmem_full[a], 1);
       mbar_init(&tmem_empty[a], kEpiWarps);
     }
     mbar_init(mma_done, 1);
+    mbar_init(sf_done, 1);
     *abort_flag = 0;
     mbar_fence_init();
   }
@@ -140,14 +156,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
   tc_fence_before();
-  __syncthreads();
+  if (kCM > 1)
+    cluster_sync();   // peers' barriers exist before any multicast reaches them
+  else
+    __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const WaitCtl ctl{abort_flag, p.err, p.timeout_ns};
 
   const int tiles_m = (int)((p.M + kBM - 1) / kBM);
   const int tiles_n = (int)((p.N + kBN - 1) / kBN);
-  const int num_tiles = tiles_m * tiles_n;
+  const int groups_m = (tiles_m + kCM - 1) / kCM;
+  const int num_ctiles = groups_m * tiles_n;
+  const int cid = (int)blockIdx.x / kCM;
+  const int ncl = (int)gridDim.x / kCM;
   const int64_t k_bytes = kFp4 ? p.K / 2 : p.K;
   const int num_kb = (int)((k_bytes + kRowBytes - 1) / kRowBytes);
   const int k_steps = (int)(k_bytes / 32);
@@ -160,8 +182,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t phase = 0;
       int issued = 0;
       const int n_atom_rows = (int)((p.N + 127) / 128);
-      for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
-        const int mb = tile % tiles_m, nb = tile / tiles_m;
+      for (int ct = cid; ct < num_ctiles; ct += ncl) {
+        const int nb = ct / groups_m;
+        const int mb = (ct % groups_m) * kCM + rank;
+        const bool m_live = mb < tiles_m;   // the last group may be partly past M
         bool ok = true;
         for (int kb = 0; kb < num_kb; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, ctl)) {
@@ -175,21 +199,30 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (kFp4) {
             nat = min(kStepsPerStage, k_steps - kb * kStepsPerStage);
             nsfb = min(C::kSfbAtoms, n_atom_rows - nb * (kBN / 128));
-            bytes += (uint32_t)(nat * 512 * (1 + nsfb));
+            bytes += (uint32_t)(nat * 512 * ((m_live ? 1 : 0) + nsfb));
           }
           mbar_arrive_expect_tx(&full[stage], bytes);
           tma_load_2d(sA, &tmap_a, &full[stage], kb * kRowBytes, mb * kBM);
-          tma_load_2d(sB, &tmap_b, &full[stage], kb * kRowBytes, nb * kBN);
+          if (kCM == 1)
+            tma_load_2d(sB, &tmap_b, &full[stage], kb * kRowBytes, nb * kBN);
+          else
+            tma_load_2d_mc(sB + rank * kBRows * kRowBytes, &tmap_b, &full[stage], kb * kRowBytes,
+                           nb * kBN + rank * kBRows, kMask);
           if (kFp4) {
             uint8_t* sSFA = sB + C::kBBytes;
             uint8_t* sSFB = sSFA + C::kSfaBytes;
-            bulk_load(sSFA, p.sfa + ((int64_t)mb * k_atoms + kb * kStepsPerStage) * 512,
-                      (uint32_t)nat * 512, &full[stage]);
-            for (int r = 0; r < nsfb; ++r)
-              bulk_load(sSFB + r * kStepsPerStage * 512,
-                        p.sfb + ((int64_t)(nb * (kBN / 128) + r) * k_atoms +
-                                 kb * kStepsPerStage) * 512,
+            if (m_live)
+              bulk_load(sSFA, p.sfa + ((int64_t)mb * k_atoms + kb * kStepsPerStage) * 512,
                         (uint32_t)nat * 512, &full[stage]);
+            for (int r = 0; r < nsfb; ++r) {
+              const uint8_t* src =
+                  p.sfb + ((int64_t)(nb * (kBN / 128) + r) * k_atoms + kb * kStepsPerStage) * 512;
+              if (kCM == 1)
+                bulk_load(sSFB + r * kStepsPerStage * 512, src, (uint32_t)nat * 512, &full[stage]);
+              else if (r % kCM == rank)
+                bulk_load_mc(sSFB + r * kStepsPerStage * 512, src, (uint32_t)nat * 512,
+                             &full[stage], kMask);
+            }
           }
           ++issued;
           if (++stage == C::kStages) {
@@ -199,8 +232,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!ok) break;
       }
-      // Wait for the last copies issued (normally complete long ago) so none
-      // is in flight when the CTA exits.
+      // Wait for the last copies into this CTA (normally complete long ago)
+      // so none is in flight when the CTA exits.
       const int n_drain = min(issued, C::kStages);
       for (int i = 0; i < n_drain; ++i) {
         if (--stage < 0) {
@@ -219,12 +252,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+      for (int ct = cid; ct < num_ctiles && ok; ct += ncl) {
         if (!mbar_wait(&tmem_empty[acc], acc_phase ^ 1u, ctl)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * kBN);
         for (int kb = 0; kb < num_kb; ++kb) {
-          if (!mbar_wait(&full[stage], phase, ctl)) {
+          if (!mbar_wait(&full[stage], phase, ctl) ||
+              (kFp4 && !mbar_wait(&sf_ready[stage], phase, ctl))) {
             ok = false;
             break;
           }
@@ -237,23 +271,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t bdesc = sdesc_k128(sB + j * 32);
             const uint32_t accumulate = (kb > 0 || j > 0) ? 1u : 0u;
             if (kFp4) {
-              const uint32_t sSFA = sB + C::kBBytes;
-              const uint32_t sSFB = sSFA + C::kSfaBytes;
               const uint32_t sfa_t = tmem_base + (uint32_t)(C::kSfColBase +
                                                             (stage * kStepsPerStage + j) *
                                                                 C::kSfColsPerStep);
-              const uint32_t sfb_t = sfa_t + 4;
-              tc_cp_scales(sfa_t, sdesc_scales(sSFA + j * 512));
-#pragma unroll
-              for (int r = 0; r < C::kSfbAtoms; ++r)
-                tc_cp_scales(sfb_t + 4 * r,
-                             sdesc_scales(sSFB + r * kStepsPerStage * 512 + j * 512));
-              mma_nvfp4(d_tmem, adesc, bdesc, idesc, sfa_t, sfb_t, accumulate);
+              mma_nvfp4(d_tmem, adesc, bdesc, idesc, sfa_t, sfa_t + 4, accumulate);
             } else {
               mma_fp8(d_tmem, adesc, bdesc, idesc, accumulate);
             }
           }
-          tc_commit(&empty[stage]);
+          // the stage is free once this CTA's MMAs have read it: tell every
+          // CTA of the cluster (their producers multicast into it)
+          if (kCM == 1)
+            tc_commit(&empty[stage]);
+          else
+            tc_commit_mc(&empty[stage], kMask);
           if (++stage == C::kStages) {
             stage = 0;
             phase ^= 1u;
@@ -272,51 +303,111 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_commit(mma_done);
       mbar_drain(mma_done, 0, p.timeout_ns, p.err);
     }
+  } else if (warp == 2) {
+    // --------------------------------------------- NVFP4 scale copies ---
+    // Block scales move shared -> TMEM from their own thread, so the copies
+    // run beside the MMA stream instead of in it.
+    if (kFp4 && lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int ct = cid; ct < num_ctiles; ct += ncl) {
+        bool ok = true;
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait(&full[stage], phase, ctl)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sSFA = smem_u32(smem + stage * C::kStageBytes) + C::kABytes + C::kBBytes;
+          const uint32_t sSFB = sSFA + C::kSfaBytes;
+          const int nsteps = min(kStepsPerStage, k_steps - kb * kStepsPerStage);
+          for (int j = 0; j < nsteps; ++j) {
+            const uint32_t sfa_t = tmem_base + (uint32_t)(C::kSfColBase +
+                                                          (stage * kStepsPerStage + j) *
+                                                              C::kSfColsPerStep);
+            tc_cp_scales(sfa_t, sdesc_scales(sSFA + j * 512));
+#pragma unroll
+            for (int r = 0; r < C::kSfbAtoms; ++r)
+              tc_cp_scales(sfa_t + 4 + 4 * r,
+                           sdesc_scales(sSFB + r * kStepsPerStage * 512 + j * 512));
+          }
+          tc_commit(&sf_ready[stage]);
+          if (++stage == C::kStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+      }
+      tc_commit(sf_done);
+      mbar_drain(sf_done, 0, p.timeout_ns, p.err);
+    }
   } else {
     // --------------------------------------------------------- epilogue ---
     constexpr int kCols = kBN / 2;  // columns per thread
     constexpr int kChunks = kCols / 32;
-    const int e = warp - 2;
+    const int e = warp - kEpiWarp0;
     const int quarter = warp & 3;   // the TMEM lane quarter this warp may access
     const int half = e >> 2;
+    uint8_t* const out_buf = out_stage + e * 4096;   // this warp's two staging boxes
     const float sdec_a = *p.sdec_a;
     const float alpha = kFp4 ? __fmul_rn(sdec_a, *p.sdec_w) : 0.0f;
     float s_enc_next = 0.0f;
     if (kRequant) {
       const float s_next = *p.next_scale;
       s_enc_next = encode_scale(s_next);
-      if (blockIdx.x == 0 && threadIdx.x == 64 && p.rq_tensor_scale != p.next_scale)
+      if (blockIdx.x == 0 && threadIdx.x == kEpiWarp0 * 32 && p.rq_tensor_scale != p.next_scale)
         *p.rq_tensor_scale = s_next;
     }
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+    for (int ct = cid; ct < num_ctiles; ct += ncl) {
       if (!mbar_wait(&tmem_full[acc], acc_phase, ctl)) break;
       tc_fence_after();
-      const int mb = tile % tiles_m, nb = tile / tiles_m;
+      const int nb = ct / groups_m;
+      const int mb = (ct % groups_m) * kCM + rank;
       const int64_t row = (int64_t)mb * kBM + quarter * 32 + lane;
       const int64_t col0 = (int64_t)nb * kBN + half * kCols;
       uint32_t packed[kCols / 2];
       const uint32_t taddr =
           tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * kBN + half * kCols);
 #pragma unroll
-      for (int c = 0; c < kChunks; ++c) {
-        uint32_t r[32];
-        tmem_ld32(taddr + c * 32, r);
+      for (int c2 = 0; c2 < kChunks; c2 += 2) {
+        // two 32-column loads in flight per wait
+        uint32_t r[2][32];
+        tmem_ld32(taddr + c2 * 32, r[0]);
+        tmem_ld32(taddr + c2 * 32 + 32, r[1]);
         tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          float a0 = alpha, a1 = alpha;
-          if (!kFp4) {
-            const int64_t n = col0 + c * 32 + 2 * i;
-            const float w0 = p.w_per_channel ? (n < p.N ? __ldg(p.sdec_w + n) : 0.0f) : *p.sdec_w;
-            const float w1 =
-                p.w_per_channel ? (n + 1 < p.N ? __ldg(p.sdec_w + n + 1) : 0.0f) : *p.sdec_w;
-            a0 = __fmul_rn(sdec_a, w0);
-            a1 = __fmul_rn(sdec_a, w1);
+        for (int h = 0; h < 2; ++h) {
+          const int c = c2 + h;
+          float a[32];
+          if (kFp4) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) a[i] = alpha;
+          } else {
+            const int64_t n0 = col0 + c * 32;
+            if (p.w_per_channel && n0 < p.N) {
+              const float4* sw = reinterpret_cast<const float4*>(p.sdec_w + n0);
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                const float4 v = __ldg(sw + i);
+                a[4 * i] = __fmul_rn(sdec_a, v.x);
+                a[4 * i + 1] = __fmul_rn(sdec_a, v.y);
+                a[4 * i + 2] = __fmul_rn(sdec_a, v.z);
+                a[4 * i + 3] = __fmul_rn(sdec_a, v.w);
+              }
+            } else {
+              const float a0 = p.w_per_channel ? 0.0f : __fmul_rn(sdec_a, *p.sdec_w);
+#pragma unroll
+              for (int i = 0; i < 32; ++i) a[i] = a0;
+            }
           }
-          packed[c * 16 + i] = pack_bf16x2(__fmul_rn(__uint_as_float(r[2 * i]), a0),
-                                           __fmul_rn(__uint_as_float(r[2 * i + 1]), a1));
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            packed[c * 16 + i] =
+                pack_bf16x2(__fmul_rn(__uint_as_float(r[h][2 * i]), a[2 * i]),
+                            __fmul_rn(__uint_as_float(r[h][2 * i + 1]), a[2 * i + 1]));
         }
       }
       // The accumulator is in registers: hand it back to the MMA warp.
@@ -330,15 +421,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         acc_phase ^= 1u;
       }
 
-      if (row < p.M) {
-        if (p.y != nullptr) {
-          uint16_t* yr = p.y + row * p.N + col0;
+      if (p.y != nullptr) {
+        // bf16 output: each 32 x 32 box goes through a 64-byte-swizzled
+        // staging buffer and one TMA store (rows >= M, cols >= N are clipped).
 #pragma unroll
-          for (int v = 0; v < kCols / 8; ++v)
-            if (col0 + v * 8 < p.N)
-              st_global_v4(yr + v * 8, packed[4 * v], packed[4 * v + 1], packed[4 * v + 2],
-                           packed[4 * v + 3]);
+        for (int c = 0; c < kChunks; ++c) {
+          uint8_t* const bufp = out_buf + (c & 1) * 2048;
+          const uint32_t buf = smem_u32(bufp);
+          if (lane == 0) bulk_wait_group_read<1>();   // this buffer's last store has read it
+          __syncwarp();
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            st_shared_v4(buf + lane * 64 + ((k ^ ((lane >> 1) & 3)) << 4), packed[c * 16 + 4 * k],
+                         packed[c * 16 + 4 * k + 1], packed[c * 16 + 4 * k + 2],
+                         packed[c * 16 + 4 * k + 3]);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tmap_y, bufp, (int32_t)(col0 + c * 32), (int32_t)(row - lane));
+            bulk_commit_group();
+          }
         }
+      }
+      if (row < p.M) {
         if (kRequant) {
 #pragma unroll
           for (int g = 0; g < kCols / 64; ++g) {
@@ -376,9 +481,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+    if (lane == 0) bulk_wait_group_all();   // output stores complete before exit
   }
 
-  __syncthreads();
+  // No CTA of the cluster may exit while a peer can still multicast into it
+  // or arrive on its barriers.
+  tc_fence_before();
+  if (kCM > 1)
+    cluster_sync();
+  else
+    __syncthreads();
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, C::kTmemCols);
@@ -421,16 +533,19 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-template <bool kFp4, int kBN, bool kRequant>
+template <bool kFp4, int kBN, int kCM, bool kRequant>
 cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned* err,
                        uint64_t timeout_ns) {
   using C = Cfg<kFp4, kBN>;
   const uint64_t k_bytes = kFp4 ? (uint64_t)a.K / 2 : (uint64_t)a.K;
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, ty;
+  std::memset(&ty, 0, sizeof ty);
   if (encode_tensor_map_2d_u8(&ta, a.a_codes, k_bytes, (uint64_t)a.M, kRowBytes, kBM) !=
           CUDA_SUCCESS ||
-      encode_tensor_map_2d_u8(&tb, a.w_codes, k_bytes, (uint64_t)a.N, kRowBytes, kBN) !=
-          CUDA_SUCCESS)
+      encode_tensor_map_2d_u8(&tb, a.w_codes, k_bytes, (uint64_t)a.N, kRowBytes, kBN / kCM) !=
+          CUDA_SUCCESS ||
+      (a.y != nullptr && encode_tensor_map_out_bf16(&ty, a.y, (uint64_t)a.N, (uint64_t)a.M) !=
+                             CUDA_SUCCESS))
     return cudaErrorInvalidValue;
   KParams p{};
   p.sfa = a.sfa;
@@ -450,33 +565,55 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   p.rq_cols = a.rq_cols;
   p.err = err;
   p.timeout_ns = timeout_ns;
-  auto kern = gemm_kernel<kFp4, kBN, kRequant>;
-  static std::once_flag attr_once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(attr_once, [&] {
-    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    C::kSmemBytes);
+  auto kern = gemm_kernel<kFp4, kBN, kCM, kRequant>;
+
+  cudaLaunchConfig_t cfg{};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kCM;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+
+  // one-time per instantiation: opt into the shared memory size and find how
+  // many clusters fit at once (a persistent grid never exceeds that)
+  static std::once_flag once;
+  static cudaError_t setup_err = cudaSuccess;
+  static int max_clusters = 0;
+  std::call_once(once, [&] {
+    setup_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     C::kSmemBytes);
+    if (setup_err != cudaSuccess) return;
+    cfg.gridDim = dim3((unsigned)(num_sms / kCM * kCM), 1, 1);
+    setup_err = cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg);
+    if (setup_err == cudaSuccess && max_clusters < 1) setup_err = cudaErrorInvalidConfiguration;
   });
-  if (attr_err != cudaSuccess) return attr_err;
-  const int64_t tiles = ((a.M + kBM - 1) / kBM) * ((a.N + kBN - 1) / kBN);
-  const int grid = (int)std::min<int64_t>(tiles, num_sms);
-  kern<<<grid, kThreads, C::kSmemBytes, s>>>(ta, tb, p);
-  return cudaGetLastError();
+  if (setup_err != cudaSuccess) return setup_err;
+  const int64_t tiles_m = (a.M + kBM - 1) / kBM;
+  const int64_t ctiles = ((tiles_m + kCM - 1) / kCM) * ((a.N + kBN - 1) / kBN);
+  const int clusters = (int)std::min<int64_t>(ctiles, std::min(max_clusters, num_sms / kCM));
+  cfg.gridDim = dim3((unsigned)(clusters * kCM), 1, 1);
+  return cudaLaunchKernelEx(&cfg, kern, ta, tb, ty, p);
 }
 
 template <bool kFp4>
 cudaError_t dispatch_bn(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned* err,
                         uint64_t timeout_ns) {
-  // 128 x 256 tiles when they fill the machine, else 128 x 128 (small M).
+  // 128 x 256 tiles in clusters of two along M (shared weight tile) when they
+  // fill the machine, else 128 x 128 single-CTA tiles (small M).
   const int64_t tiles256 = ((a.M + kBM - 1) / kBM) * ((a.N + 255) / 256);
   const bool wide = tiles256 >= num_sms;
   if constexpr (kFp4) {
     if (a.next_scale != nullptr)
-      return wide ? launch_cfg<true, 256, true>(a, s, num_sms, err, timeout_ns)
-                  : launch_cfg<true, 128, true>(a, s, num_sms, err, timeout_ns);
+      return wide ? launch_cfg<true, 256, 2, true>(a, s, num_sms, err, timeout_ns)
+                  : launch_cfg<true, 128, 1, true>(a, s, num_sms, err, timeout_ns);
   }
-  return wide ? launch_cfg<kFp4, 256, false>(a, s, num_sms, err, timeout_ns)
-              : launch_cfg<kFp4, 128, false>(a, s, num_sms, err, timeout_ns);
+  return wide ? launch_cfg<kFp4, 256, 2, false>(a, s, num_sms, err, timeout_ns)
+              : launch_cfg<kFp4, 128, 1, false>(a, s, num_sms, err, timeout_ns);
 }
 
 }  // namespace
@@ -491,6 +628,20 @@ CUresult encode_tensor_map_2d_u8(CUtensorMap* map, const void* base, uint64_t in
   const cuuint32_t estr[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+// bf16 [rows, cols] output map: 32 x 32 boxes, 64-byte swizzle (the layout of
+// the epilogue's staging boxes).
+CUresult encode_tensor_map_out_bf16(CUtensorMap* map, void* base, uint64_t cols, uint64_t rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (fn == nullptr) return CUDA_ERROR_NOT_FOUND;
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {cols * 2};
+  const cuuint32_t box[2] = {32, 32};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 

@@ -47,6 +47,7 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned
 cudaError_t launch_wait_selftest(uint64_t timeout_ns, cudaStream_t s, unsigned* err);
 
 // Resolves cuTensorMapEncodeTiled through the runtime (no libcuda link).
+CUresult encode_tensor_map_out_bf16(CUtensorMap* map, void* base, uint64_t cols, uint64_t rows);
 CUresult encode_tensor_map_2d_u8(CUtensorMap* map, const void* base, uint64_t inner_bytes,
                                  uint64_t rows, uint32_t box_inner, uint32_t box_rows);
 
