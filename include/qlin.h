@@ -192,6 +192,37 @@ qlin_status qlin_linear_fused(const qlin_nvfp4_t *A, const qlin_nvfp4_t *W,
                               void *y_bf16, const float *next_scale,
                               qlin_nvfp4_t *y_q, int64_t rq_col0, void *stream);
 
+/* Bytes of device scratch that qlin_quantize_act_nvfp4_noalloc keeps in the
+ * library's own static device array (per GPU that loads the library). */
+#define QLIN_NOALLOC_SCRATCH_BYTES 256
+
+/*
+ * qlin_quantize_act_nvfp4 with the dynamic tensor scale, for callers that
+ * cannot allocate device memory.  The paper has no counterpart: it is an
+ * integration aid.  Some callers own no allocator of their own -- a plugin
+ * running inside an inference runtime that hands out all device memory, or a
+ * real-time loop that must never stall on cudaMalloc.  They can still pass x
+ * and the output buffers, but not the workspace the dynamic amax pass needs.
+ *
+ * This entry point takes no workspace: its scratch (the amax word) lives in a
+ * static device array of QLIN_NOALLOC_SCRATCH_BYTES bytes that the library
+ * holds on every GPU that loads it, until the process exits.  It calls no
+ * cudaMalloc, cudaFree or other allocating routine.
+ *  - x, M, K, out: as for qlin_quantize_act_nvfp4 (out->tensor_scale receives
+ *    the dynamic S_dec = amax / 2688).
+ *  - The first call on a device looks up the array's device address
+ *    (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture.
+ *  - Every call shares the one array and clears the part it uses before use.
+ *    Calls whose work overlaps on the GPU (different streams, no ordering)
+ *    race on it: order them on one stream or serialise them.
+ *  - Returns QLIN_ERR_WORKSPACE if the scratch a shape needs
+ *    (qlin_workspace_size(M, K)) exceeds QLIN_NOALLOC_SCRATCH_BYTES; other
+ *    errors as for qlin_quantize_act_nvfp4.
+ */
+qlin_status qlin_quantize_act_nvfp4_noalloc(const void *x_bf16, int64_t M, int64_t K,
+                                            qlin_nvfp4_t *out, void *stream);
+
 /*
  * Waits for `stream`, then returns and clears the device status word:
  * QLIN_ERR_TIMEOUT if a kernel's bounded wait expired since the last call,

@@ -55,6 +55,27 @@ qlin_status device_state(unsigned** status, int* num_sms) {
   return QLIN_OK;
 }
 
+// Scratch of qlin_quantize_act_nvfp4_noalloc: a static device array, so the
+// entry point needs no allocation.  Host code may only use its device address
+// (looked up once per device), never the symbol itself.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[QLIN_NOALLOC_SCRATCH_BYTES];
+unsigned char* g_noalloc_ptr[kMaxDevices] = {};
+
+qlin_status noalloc_scratch(unsigned char** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (dev < 0 || dev >= kMaxDevices) return QLIN_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_dev_mutex);
+  if (g_noalloc_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    if ((e = cudaGetSymbolAddress(&p, g_noalloc_scratch)) != cudaSuccess) return cuda_fail(e);
+    g_noalloc_ptr[dev] = static_cast<unsigned char*>(p);
+  }
+  *out = g_noalloc_ptr[dev];
+  return QLIN_OK;
+}
+
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 bool shape_ok(int64_t rows, int64_t K) { return rows >= 1 && K >= 64 && K % 64 == 0; }
@@ -131,6 +152,30 @@ qlin_status qlin_quantize_act_nvfp4(const void* x_bf16, int64_t M, int64_t K,
   } else {
     QLIN_CUDA(launch_quant_nvfp4(x_bf16, M, K, static_scale, false, *out, s, sms));
   }
+  return QLIN_OK;
+}
+
+qlin_status qlin_quantize_act_nvfp4_noalloc(const void* x_bf16, int64_t M, int64_t K,
+                                            qlin_nvfp4_t* out, void* stream) {
+  if (x_bf16 == nullptr || !shape_ok(M, K)) return QLIN_ERR_INVALID_ARG;
+  QLIN_TRY(check_nvfp4(out, M, K));
+  if (!aligned(x_bf16, 16)) return QLIN_ERR_MISALIGNED;
+  if (qlin_workspace_size(M, K) > QLIN_NOALLOC_SCRATCH_BYTES) {
+    std::snprintf(g_last_error, sizeof g_last_error,
+                  "shape [%lld, %lld] needs more than %d bytes of static scratch",
+                  (long long)M, (long long)K, QLIN_NOALLOC_SCRATCH_BYTES);
+    return QLIN_ERR_WORKSPACE;
+  }
+  unsigned* status;
+  int sms;
+  QLIN_TRY(device_state(&status, &sms));
+  unsigned char* scratch = nullptr;
+  QLIN_TRY(noalloc_scratch(&scratch));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unsigned* amax = reinterpret_cast<unsigned*>(scratch);  // cleared by launch_amax
+  QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms));
+  QLIN_CUDA(launch_quant_nvfp4(x_bf16, M, K, reinterpret_cast<const float*>(amax), true, *out, s,
+                               sms));
   return QLIN_OK;
 }
 

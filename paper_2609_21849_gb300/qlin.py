@@ -24,7 +24,7 @@ STATUS = {0: "QLIN_OK", 1: "QLIN_ERR_INVALID_ARG", 2: "QLIN_ERR_UNSUPPORTED",
 # Every function declared in include/qlin.h.
 EXPORTS = ("qlin_nvfp4_scale_bytes", "qlin_workspace_size", "qlin_quantize_act_nvfp4",
            "qlin_quantize_act_fp8", "qlin_quantize_weight", "qlin_gemm_nvfp4", "qlin_gemm_fp8",
-           "qlin_linear_fused", "qlin_sync_status", "qlin_selftest_bounded_wait",
+           "qlin_linear_fused", "qlin_quantize_act_nvfp4_noalloc", "qlin_sync_status", "qlin_selftest_bounded_wait",
            "qlin_set_wait_timeout_ns", "qlin_status_str", "qlin_last_error")
 
 
@@ -71,6 +71,7 @@ def load_library(path: str = LIB_PATH):
             "qlin_gemm_fp8": (ctypes.c_int, [ctypes.POINTER(FP8Desc), ctypes.POINTER(FP8Desc), p, p]),
             "qlin_linear_fused": (ctypes.c_int, [ctypes.POINTER(NVFP4Desc), ctypes.POINTER(NVFP4Desc), p, p,
                                                  ctypes.POINTER(NVFP4Desc), i64, p]),
+            "qlin_quantize_act_nvfp4_noalloc": (ctypes.c_int, [p, i64, i64, ctypes.POINTER(NVFP4Desc), p]),
             "qlin_sync_status": (ctypes.c_int, [p]),
             "qlin_selftest_bounded_wait": (ctypes.c_int, [ctypes.c_uint64, p]),
             "qlin_set_wait_timeout_ns": (None, [ctypes.c_uint64]),
@@ -186,6 +187,20 @@ def qlin_quantize_act_nvfp4(x: torch.Tensor, static_scale: torch.Tensor | None =
     _check(load_library().qlin_quantize_act_nvfp4(
         _ptr(x), M, K, _ptr(static_scale), ctypes.byref(d), _ptr(workspace),
         0 if workspace is None else workspace.numel(), _stream(stream)), "qlin_quantize_act_nvfp4")
+    return out
+
+
+def qlin_quantize_act_nvfp4_noalloc(x: torch.Tensor, out: NVFP4Tensor, stream=None) -> NVFP4Tensor:
+    """Dynamic-scale NVFP4 quantization for callers that cannot allocate device
+    memory: no workspace argument; the library keeps the amax scratch in its
+    own static device array.  ``out`` must be supplied by the caller.  Calls
+    that overlap on the GPU share that scratch and race; the first call on a
+    device should come before any stream capture."""
+    M, K = _bf16_2d(x)
+    d = out.desc()
+    _check(load_library().qlin_quantize_act_nvfp4_noalloc(_ptr(x), M, K, ctypes.byref(d),
+                                                          _stream(stream)),
+           "qlin_quantize_act_nvfp4_noalloc")
     return out
 
 
