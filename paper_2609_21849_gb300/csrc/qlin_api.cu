@@ -76,6 +76,8 @@ qlin_status noalloc_scratch(unsigned char** out) {
   return QLIN_OK;
 }
 
+uint64_t timeout() { return g_timeout_ns.load(std::memory_order_relaxed); }
+
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 bool shape_ok(int64_t rows, int64_t K) { return rows >= 1 && K >= 64 && K % 64 == 0; }
@@ -146,11 +148,11 @@ qlin_status qlin_quantize_act_nvfp4(const void* x_bf16, int64_t M, int64_t K,
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (static_scale == nullptr) {
     unsigned* amax = static_cast<unsigned*>(workspace);
-    QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms));
+    QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms, status, timeout()));
     QLIN_CUDA(launch_quant_nvfp4(x_bf16, M, K, reinterpret_cast<const float*>(amax), true, *out,
-                                 s, sms));
+                                 s, sms, status, timeout()));
   } else {
-    QLIN_CUDA(launch_quant_nvfp4(x_bf16, M, K, static_scale, false, *out, s, sms));
+    QLIN_CUDA(launch_quant_nvfp4(x_bf16, M, K, static_scale, false, *out, s, sms, status, timeout()));
   }
   return QLIN_OK;
 }
@@ -173,9 +175,9 @@ qlin_status qlin_quantize_act_nvfp4_noalloc(const void* x_bf16, int64_t M, int64
   QLIN_TRY(noalloc_scratch(&scratch));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   unsigned* amax = reinterpret_cast<unsigned*>(scratch);  // cleared by launch_amax
-  QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms));
+  QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms, status, timeout()));
   QLIN_CUDA(launch_quant_nvfp4(x_bf16, M, K, reinterpret_cast<const float*>(amax), true, *out, s,
-                               sms));
+                               sms, status, timeout()));
   return QLIN_OK;
 }
 
@@ -194,11 +196,11 @@ qlin_status qlin_quantize_act_fp8(const void* x_bf16, int64_t M, int64_t K,
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (static_scale == nullptr) {
     unsigned* amax = static_cast<unsigned*>(workspace);
-    QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms));
+    QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms, status, timeout()));
     QLIN_CUDA(launch_quant_fp8(x_bf16, M, K, reinterpret_cast<const float*>(amax), true, *out, s,
-                               sms));
+                               sms, status, timeout()));
   } else {
-    QLIN_CUDA(launch_quant_fp8(x_bf16, M, K, static_scale, false, *out, s, sms));
+    QLIN_CUDA(launch_quant_fp8(x_bf16, M, K, static_scale, false, *out, s, sms, status, timeout()));
   }
   return QLIN_OK;
 }

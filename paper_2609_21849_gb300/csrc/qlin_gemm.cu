@@ -33,7 +33,7 @@ constexpr int kBM = 128;
 constexpr int kRowBytes = 128;      // bytes of K per stage and row: one swizzle row
 constexpr int kStepsPerStage = 4;   // one MMA per 32 bytes of K
 constexpr int kEpiWarps = 8;
-constexpr int kEpiWarp0 = 3;                      // warps 0-2: producer, MMA, scale copies
+constexpr int kEpiWarp0 = 4;   // warps 0-3: producer, MMA, two scale-copy warps
 constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
 constexpr int kSmemBudget = 232448 - 2048;  // opt-in shared memory minus barriers/alignment
 
@@ -124,11 +124,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* full = reinterpret_cast<uint64_t*>(out_stage + C::kOutBytes);
   uint64_t* empty = full + C::kStages;
   uint64_t* sf_ready = empty + C::kStages;   // NVFP4: the stage's scales are in TMEM
-  uint64_t* tmem_full = sf_ready + C::kStages;
+  uint64_t* sf_full = sf_ready + C::kStages;  // NVFP4: the stage's scale bytes landed
+  uint64_t* tmem_full = sf_full + C::kStages;
   uint64_t* tmem_empty = tmem_full + 2;
   uint64_t* mma_done = tmem_empty + 2;
-  uint64_t* sf_done = mma_done + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sf_done + 1);
+  uint64_t* sf_done = mma_done + 1;   // two barriers, one per scale-copy warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sf_done + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -139,14 +140,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], kCM);   // one arrival from the MMA warp of each CTA
-      mbar_init(&sf_ready[s], 1);
+      mbar_init(&sf_ready[s], 2);   // one commit per scale-copy warp
+      mbar_init(&sf_full[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tmem_full[a], 1);
       mbar_init(&tmem_empty[a], kEpiWarps);
     }
     mbar_init(mma_done, 1);
-    mbar_init(sf_done, 1);
+    mbar_init(&sf_done[0], 1);
+    mbar_init(&sf_done[1], 1);
     *abort_flag = 0;
     mbar_fence_init();
   }
@@ -177,11 +180,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------ TMA producer ---
-    if (lane == 0) {
+    // A TMA instruction occupies its issuing thread for hundreds of cycles,
+    // so the stage's copies are issued by several lanes executing the SAME
+    // instruction with per-lane operands: lanes 0 and 1 one tensor load (A
+    // tile, W tile), lanes 2.. one bulk copy (A scales, W scale rows).
+    const int nlanes = kFp4 ? 3 + C::kSfbAtoms : 2;
+    if (lane < nlanes) {
       int stage = 0;
       uint32_t phase = 0;
       int issued = 0;
       const int n_atom_rows = (int)((p.N + 127) / 128);
+      const uint16_t self_mask = (uint16_t)(1u << rank);
       for (int ct = cid; ct < num_ctiles; ct += ncl) {
         const int nb = ct / groups_m;
         const int mb = (ct % groups_m) * kCM + rank;
@@ -194,34 +203,41 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           uint8_t* sA = smem + stage * C::kStageBytes;
           uint8_t* sB = sA + C::kABytes;
-          uint32_t bytes = C::kABytes + C::kBBytes;
-          int nat = 0, nsfb = 0;
-          if (kFp4) {
-            nat = min(kStepsPerStage, k_steps - kb * kStepsPerStage);
-            nsfb = min(C::kSfbAtoms, n_atom_rows - nb * (kBN / 128));
-            bytes += (uint32_t)(nat * 512 * ((m_live ? 1 : 0) + nsfb));
-          }
-          mbar_arrive_expect_tx(&full[stage], bytes);
-          tma_load_2d(sA, &tmap_a, &full[stage], kb * kRowBytes, mb * kBM);
-          if (kCM == 1)
-            tma_load_2d(sB, &tmap_b, &full[stage], kb * kRowBytes, nb * kBN);
-          else
-            tma_load_2d_mc(sB + rank * kBRows * kRowBytes, &tmap_b, &full[stage], kb * kRowBytes,
-                           nb * kBN + rank * kBRows, kMask);
-          if (kFp4) {
-            uint8_t* sSFA = sB + C::kBBytes;
-            uint8_t* sSFB = sSFA + C::kSfaBytes;
-            if (m_live)
-              bulk_load(sSFA, p.sfa + ((int64_t)mb * k_atoms + kb * kStepsPerStage) * 512,
-                        (uint32_t)nat * 512, &full[stage]);
-            for (int r = 0; r < nsfb; ++r) {
-              const uint8_t* src =
-                  p.sfb + ((int64_t)(nb * (kBN / 128) + r) * k_atoms + kb * kStepsPerStage) * 512;
+          const int nat = min(kStepsPerStage, k_steps - kb * kStepsPerStage);
+          const int nsfb = kFp4 ? min(C::kSfbAtoms, n_atom_rows - nb * (kBN / 128)) : 0;
+          if (lane == 0) mbar_arrive_expect_tx(&full[stage], C::kABytes + C::kBBytes);
+          if (kFp4 && lane == 2)   // the scales complete on their own barrier
+            mbar_arrive_expect_tx(&sf_full[stage],
+                                  (uint32_t)(nat * 512 * ((m_live ? 1 : 0) + nsfb)));
+          __syncwarp((1u << nlanes) - 1u);
+          // operand tiles
+          if (lane < 2) {
+            const bool is_a = lane == 0;
+            const CUtensorMap* map = is_a ? &tmap_a : &tmap_b;
+            const int32_t y = is_a ? mb * kBM : nb * kBN + rank * kBRows;
+            uint8_t* dst = is_a ? sA : sB + rank * kBRows * kRowBytes;
+            if (kCM == 1)
+              tma_load_2d(dst, map, &full[stage], kb * kRowBytes, y);
+            else
+              tma_load_2d_mc(dst, map, &full[stage], kb * kRowBytes, y,
+                             is_a ? self_mask : kMask);
+          } else if (kFp4) {
+            // block scales: lane 2 the A atoms, lane 3 + r the W atom row r
+            const bool is_a = lane == 2;
+            const int r = lane - 3;
+            const bool live = is_a ? m_live : (r < nsfb && r % kCM == rank);
+            const uint8_t* src =
+                is_a ? p.sfa + ((int64_t)mb * k_atoms + kb * kStepsPerStage) * 512
+                     : p.sfb + ((int64_t)(nb * (kBN / 128) + r) * k_atoms + kb * kStepsPerStage) *
+                                   512;
+            uint8_t* dst = is_a ? sB + C::kBBytes
+                                : sB + C::kBBytes + C::kSfaBytes + r * kStepsPerStage * 512;
+            if (live) {
               if (kCM == 1)
-                bulk_load(sSFB + r * kStepsPerStage * 512, src, (uint32_t)nat * 512, &full[stage]);
-              else if (r % kCM == rank)
-                bulk_load_mc(sSFB + r * kStepsPerStage * 512, src, (uint32_t)nat * 512,
-                             &full[stage], kMask);
+                bulk_load(dst, src, (uint32_t)nat * 512, &sf_full[stage]);
+              else
+                bulk_load_mc(dst, src, (uint32_t)nat * 512, &sf_full[stage],
+                             is_a ? self_mask : kMask);
             }
           }
           ++issued;
@@ -234,13 +250,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // Wait for the last copies into this CTA (normally complete long ago)
       // so none is in flight when the CTA exits.
-      const int n_drain = min(issued, C::kStages);
-      for (int i = 0; i < n_drain; ++i) {
-        if (--stage < 0) {
-          stage = C::kStages - 1;
-          phase ^= 1u;
+      if (lane == 0 || (kFp4 && lane == 2)) {
+        uint64_t* bars = lane == 0 ? full : sf_full;
+        const int n_drain = min(issued, C::kStages);
+        for (int i = 0; i < n_drain; ++i) {
+          if (--stage < 0) {
+            stage = C::kStages - 1;
+            phase ^= 1u;
+          }
+          mbar_drain(&bars[stage], phase, p.timeout_ns, p.err);
         }
-        mbar_drain(&full[stage], phase, p.timeout_ns, p.err);
       }
     }
   } else if (warp == 1) {
@@ -303,17 +322,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_commit(mma_done);
       mbar_drain(mma_done, 0, p.timeout_ns, p.err);
     }
-  } else if (warp == 2) {
+  } else if (warp == 2 || warp == 3) {
     // --------------------------------------------- NVFP4 scale copies ---
-    // Block scales move shared -> TMEM from their own thread, so the copies
-    // run beside the MMA stream instead of in it.
+    // Block scales move shared -> TMEM from two threads of their own (a
+    // tcgen05.cp occupies its issuing thread ~50 cycles), beside the MMA
+    // stream: warp 2 the A atoms and W atom row 0, warp 3 W atom row 1.
     if (kFp4 && lane == 0) {
+      const int sw = warp - 2;
       int stage = 0;
       uint32_t phase = 0;
       for (int ct = cid; ct < num_ctiles; ct += ncl) {
         bool ok = true;
         for (int kb = 0; kb < num_kb; ++kb) {
-          if (!mbar_wait(&full[stage], phase, ctl)) {
+          if (!mbar_wait(&sf_full[stage], phase, ctl)) {
             ok = false;
             break;
           }
@@ -325,11 +346,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t sfa_t = tmem_base + (uint32_t)(C::kSfColBase +
                                                           (stage * kStepsPerStage + j) *
                                                               C::kSfColsPerStep);
-            tc_cp_scales(sfa_t, sdesc_scales(sSFA + j * 512));
-#pragma unroll
-            for (int r = 0; r < C::kSfbAtoms; ++r)
-              tc_cp_scales(sfa_t + 4 + 4 * r,
-                           sdesc_scales(sSFB + r * kStepsPerStage * 512 + j * 512));
+            if (sw == 0) {
+              tc_cp_scales(sfa_t, sdesc_scales(sSFA + j * 512));
+              tc_cp_scales(sfa_t + 4, sdesc_scales(sSFB + j * 512));
+            } else if (C::kSfbAtoms > 1) {
+              tc_cp_scales(sfa_t + 8, sdesc_scales(sSFB + kStepsPerStage * 512 + j * 512));
+            }
           }
           tc_commit(&sf_ready[stage]);
           if (++stage == C::kStages) {
@@ -339,8 +361,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!ok) break;
       }
-      tc_commit(sf_done);
-      mbar_drain(sf_done, 0, p.timeout_ns, p.err);
+      tc_commit(&sf_done[sw]);
+      mbar_drain(&sf_done[sw], 0, p.timeout_ns, p.err);
     }
   } else {
     // --------------------------------------------------------- epilogue ---

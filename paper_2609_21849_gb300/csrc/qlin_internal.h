@@ -13,13 +13,15 @@
 namespace qlin {
 
 // ---- quantizers (qlin_quant.cu) ----
+// err / timeout_ns: device status word and limit of the bounded waits.
 cudaError_t launch_amax(const void* x, int64_t n_elems, unsigned* amax_bits, cudaStream_t s,
-                        int num_sms);
+                        int num_sms, unsigned* err, uint64_t timeout_ns);
 cudaError_t launch_quant_nvfp4(const void* x, int64_t M, int64_t K, const float* scale_src,
                                bool dynamic, const qlin_nvfp4_t& out, cudaStream_t s,
-                               int num_sms);
+                               int num_sms, unsigned* err, uint64_t timeout_ns);
 cudaError_t launch_quant_fp8(const void* x, int64_t M, int64_t K, const float* scale_src,
-                             bool dynamic, const qlin_fp8_t& out, cudaStream_t s, int num_sms);
+                             bool dynamic, const qlin_fp8_t& out, cudaStream_t s, int num_sms,
+                             unsigned* err, uint64_t timeout_ns);
 cudaError_t launch_quant_fp8_rows(const void* w, int64_t N, int64_t K, const qlin_fp8_t& out,
                                   cudaStream_t s, int num_sms);
 

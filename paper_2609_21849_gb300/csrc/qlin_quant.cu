@@ -2,26 +2,31 @@
 // post-training quantization; activations are quantized at run time, weights
 // once).  All kernels here are HBM-bandwidth bound streaming kernels:
 //
-//   amax_bf16_kernel      max |x| over a tensor (the dynamic tensor scale)
-//   quant_nvfp4_kernel    bf16 -> packed e2m1 codes + E4M3 block scales in the
+//   amax_kernel           max |x| over a tensor (the dynamic tensor scale)
+//   quant_kernel<NVFP4>   bf16 -> packed e2m1 codes + E4M3 block scales in the
 //                         tensor-core scale layout + FP32 tensor scale
-//   quant_fp8_kernel      bf16 -> E4M3 codes with one tensor scale
+//   quant_kernel<FP8>     bf16 -> E4M3 codes with one tensor scale
 //   quant_fp8_rows_kernel bf16 weights -> E4M3 codes with one scale per row
 //
-// Data layout of the streaming kernels: the [M, K] input is viewed as a flat
-// array of 8-element (16-byte) chunks.  A warp covers 32 consecutive chunks
-// (512 contiguous bytes) per load instruction; two neighbouring lanes hold
-// one 16-element block, eight neighbouring lanes one 64-element group whose
-// four block scales form one 32-bit word of the scale layout.  Because
-// K % 64 == 0, a group never straddles a row.
+// Streaming structure: the [M, K] input is a flat array of 16-byte chunks (8
+// bf16), cut into 16 KB tiles.  A persistent grid (three CTAs per SM)
+// streams tiles through a four-deep shared-memory ring filled by bulk copies,
+// so ~192 KB per SM of input is in flight regardless of register pressure.
+// Inside a tile, each thread takes consecutive units of chunks (NVFP4: one
+// 16-element block per lane, so four neighbouring lanes hold one 64-element
+// group, whose four block scales form one 32-bit word of the scale layout;
+// because K % 64 == 0 a group never straddles a row).
 #include "qlin_internal.h"
 
 namespace qlin {
 
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kUnroll = 4;  // 16-byte chunks in flight per lane
+constexpr int kThreads = 512;
+constexpr int kTileChunks = 1024;             // 16 KB of input per tile
+constexpr int kStages = 4;
+constexpr int kSmem = kStages * kTileChunks * 16 + 64;
+constexpr int kBlocksPerSm = 3;
 
 // Largest |bf16| in a 16-byte chunk, as the bit pattern of a bf16 magnitude.
 __device__ __forceinline__ uint32_t chunk_abs_max_bits(const uint4 v) {
@@ -37,24 +42,188 @@ __device__ __forceinline__ void unpack8(const uint4 v, float (&f)[8]) {
   f[6] = bf16_lo(v.w); f[7] = bf16_hi(v.w);
 }
 
-// amax over n_chunks 16-byte chunks, folded into *amax_bits (fp32 bits;
-// must be zero before the launch).
-__global__ void __launch_bounds__(kThreads) amax_bf16_kernel(const uint4* __restrict__ x,
-                                                             int64_t n_chunks,
-                                                             unsigned* __restrict__ amax_bits) {
-  __shared__ uint32_t warp_max[kThreads / 32];
+__device__ __forceinline__ uint4 lds128(const uint4* p) {
+  uint4 v;
+  asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(smem_u32(p)));
+  return v;
+}
+
+// The per-tile work of each kernel (called by every thread for each tile).
+struct AmaxOp {
+  static constexpr int kUnit = 1;   // chunks per thread and call
   uint32_t m = 0;
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
-  int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  for (; c + (kUnroll - 1) * stride < n_chunks; c += kUnroll * stride) {
-    uint4 v[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) v[u] = __ldg(x + c + u * stride);
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) m = max(m, chunk_abs_max_bits(v[u]));
+  __device__ __forceinline__ void init() {}
+  __device__ __forceinline__ void unit(const uint4 (&v)[1], uint64_t, bool valid) {
+    if (valid) m = max(m, chunk_abs_max_bits(v[0]));
   }
-  for (; c < n_chunks; c += stride) m = max(m, chunk_abs_max_bits(__ldg(x + c)));
-  m = __reduce_max_sync(0xFFFFFFFFu, m);
+};
+
+// One lane per 16-element block (two chunks); lanes 4g..4g+3 hold the four
+// blocks of a 64-element group.  r_b = S_enc / s_b comes from a per-CTA table
+// over the 127 finite E4M3 codes, filled with the same fp32 division.
+template <typename Idx>
+struct Nvfp4Op {
+  static constexpr int kUnit = 2;
+  float s_enc;
+  Idx chunks_per_row;
+  int64_t K;
+  uint32_t* codes;
+  uint8_t* scales;
+  float* r_table;   // shared memory, 128 entries
+  __device__ __forceinline__ void init() {
+    if (threadIdx.x < 128) {
+      const uint32_t c = threadIdx.x;
+      r_table[c] = (c == 0u) ? 0.0f : __fdiv_rn(s_enc, e4m3_value(c));
+    }
+  }
+  __device__ __forceinline__ void unit(const uint4 (&v)[2], uint64_t c, bool valid) {
+    const int lane = threadIdx.x & 31;
+    const uint32_t mb = max(chunk_abs_max_bits(v[0]), chunk_abs_max_bits(v[1]));
+    const float t = __fmul_rn(__uint_as_float(mb << 16), s_enc);
+    const uint32_t sb = e4m3_code(__fdiv_rn(t, 6.0f));
+    const float r_b = r_table[sb];
+    float f[8];
+    unpack8(v[0], f);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], r_b);
+    const uint32_t code0 = e2m1x8(f);
+    unpack8(v[1], f);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], r_b);
+    const uint32_t code1 = e2m1x8(f);
+    // gather the group's four scales into its first lane
+    const uint32_t s1 = __shfl_down_sync(0xFFFFFFFFu, sb, 1);
+    const uint32_t s2 = __shfl_down_sync(0xFFFFFFFFu, sb, 2);
+    const uint32_t s3 = __shfl_down_sync(0xFFFFFFFFu, sb, 3);
+    if (valid) {
+      reinterpret_cast<uint2*>(codes)[c >> 1] = make_uint2(code0, code1);
+      if ((lane & 3) == 0) {
+        const Idx ci = (Idx)c;
+        const Idx row = ci / chunks_per_row;
+        const Idx col = (ci - row * chunks_per_row) << 3;
+        *reinterpret_cast<uint32_t*>(scales + scale_offset((int64_t)row, (int64_t)(col >> 4), K)) =
+            sb | (s1 << 8) | (s2 << 16) | (s3 << 24);
+      }
+    }
+  }
+};
+
+struct Fp8Op {
+  static constexpr int kUnit = 1;
+  float s_enc;
+  uint2* codes;
+  __device__ __forceinline__ void init() {}
+  __device__ __forceinline__ void unit(const uint4 (&v)[1], uint64_t c, bool valid) {
+    if (!valid) return;
+    float f[8];
+    unpack8(v[0], f);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], s_enc);
+    codes[c] = make_uint2(e4m3x4(f[0], f[1], f[2], f[3]), e4m3x4(f[4], f[5], f[6], f[7]));
+  }
+};
+
+// Persistent tile loop: thread 0 keeps kStages bulk copies of 16 KB tiles in
+// flight; every thread applies `op` to its chunks of each landed tile.
+// Returns false if a bounded wait expired (recorded in *err).
+template <typename Op>
+__device__ __forceinline__ bool stream_tiles(const uint4* __restrict__ x, uint64_t n_chunks,
+                                             Op& op, unsigned* err, uint64_t timeout_ns) {
+  extern __shared__ __align__(128) uint8_t qsm[];
+  uint4* buf = reinterpret_cast<uint4*>(qsm);
+  uint64_t* full = reinterpret_cast<uint64_t*>(qsm + kStages * kTileChunks * 16);
+  __shared__ int abort_flag;
+  const uint64_t n_tiles = (n_chunks + kTileChunks - 1) / kTileChunks;
+  const int tid = threadIdx.x;
+
+  auto issue = [&](uint64_t t, int s) {
+    const uint64_t c0 = t * kTileChunks;
+    const uint64_t left = n_chunks - c0;
+    const uint32_t nc = left < (uint64_t)kTileChunks ? (uint32_t)left : (uint32_t)kTileChunks;
+    mbar_arrive_expect_tx(&full[s], nc * 16u);
+    bulk_load(buf + s * kTileChunks, x + c0, nc * 16u, &full[s]);
+  };
+
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
+    abort_flag = 0;
+    mbar_fence_init();
+  }
+  op.init();
+  __syncthreads();
+  if (tid == 0)
+    for (int s = 0; s < kStages; ++s) {
+      const uint64_t t = blockIdx.x + (uint64_t)s * gridDim.x;
+      if (t < n_tiles) issue(t, s);
+    }
+  int s = 0;
+  uint32_t phase = 0;
+  bool ok = true;
+  uint64_t t_stop = 0;
+  for (uint64_t t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+    if (tid == 0) {
+      const WaitCtl ctl{&abort_flag, err, timeout_ns};
+      if (!mbar_wait(&full[s], phase, ctl)) abort_flag = 1;
+    }
+    __syncthreads();
+    if (abort_flag) {
+      ok = false;
+      t_stop = t;
+      break;
+    }
+    const uint64_t c0 = t * kTileChunks;
+    constexpr int kU = Op::kUnit;
+#pragma unroll
+    for (int u = 0; u < kTileChunks / (kU * kThreads); ++u) {
+      const int cl = (u * kThreads + tid) * kU;   // first chunk of this thread's unit
+      const uint64_t c = c0 + cl;
+      const bool valid = c < n_chunks;           // units never straddle n_chunks
+      uint4 v[kU];
+#pragma unroll
+      for (int k = 0; k < kU; ++k)
+        v[k] = valid ? lds128(buf + s * kTileChunks + cl + k) : make_uint4(0u, 0u, 0u, 0u);
+      op.unit(v, c, valid);
+    }
+    __syncthreads();   // every thread is done with this stage
+    if (tid == 0) {
+      const uint64_t nt = t + (uint64_t)kStages * gridDim.x;
+      if (nt < n_tiles) issue(nt, s);
+    }
+    if (++s == kStages) {
+      s = 0;
+      phase ^= 1u;
+    }
+  }
+  if (!ok && tid == 0) {
+    // Let every copy already issued land before the CTA exits: the tiles
+    // t_stop, t_stop + G, ... (at most kStages of them) sit in stages
+    // s, s + 1, ... with the current phase, flipping on wrap-around.
+    uint64_t tt = t_stop;
+    for (int i = 0; i < kStages && tt < n_tiles; ++i, tt += gridDim.x) {
+      const uint32_t a = smem_u32(&full[s]);
+      const uint64_t t0 = global_timer_ns();
+      while (!mbar_try_wait(a, phase) && global_timer_ns() - t0 < timeout_ns) {
+      }
+      if (++s == kStages) {
+        s = 0;
+        phase ^= 1u;
+      }
+    }
+  }
+  return ok;
+}
+
+// amax over n_chunks 16-byte chunks, folded into *amax_bits (fp32 bits;
+// cleared before the launch).
+__global__ void __launch_bounds__(kThreads, kBlocksPerSm)
+    amax_kernel(const uint4* __restrict__ x, uint64_t n_chunks, unsigned* __restrict__ amax_bits,
+                unsigned* err, uint64_t timeout_ns) {
+  __shared__ uint32_t warp_max[kThreads / 32];
+  AmaxOp op;
+  stream_tiles(x, n_chunks, op, err, timeout_ns);
+  const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, op.m);
   if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -65,92 +234,51 @@ __global__ void __launch_bounds__(kThreads) amax_bf16_kernel(const uint4* __rest
   }
 }
 
-// NVFP4 quantizer.  kDynamic: scale_src holds amax (fp32) and
-// S_dec = amax / 2688 (1 if amax == 0); otherwise scale_src holds S_dec.
+// Tensor scale: kDynamic -> scale_src holds amax, S_dec = amax / qmax (1 if
+// amax == 0); otherwise scale_src holds S_dec.  Block 0 records S_dec.
 template <bool kDynamic>
-__global__ void __launch_bounds__(kThreads) quant_nvfp4_kernel(
-    const uint4* __restrict__ x, int64_t n_chunks, int64_t K, const float* scale_src,
-    float* sdec_out, uint32_t* __restrict__ codes, uint8_t* __restrict__ scales) {
+__device__ __forceinline__ float tensor_scale(const float* scale_src, float* sdec_out,
+                                              float qmax) {
   float s_dec;
   if (kDynamic) {
     const float amax = *scale_src;
-    s_dec = (amax == 0.0f) ? 1.0f : __fdiv_rn(amax, 2688.0f);
+    s_dec = (amax == 0.0f) ? 1.0f : __fdiv_rn(amax, qmax);
   } else {
     s_dec = *scale_src;
   }
-  const float s_enc = encode_scale(s_dec);
   if (blockIdx.x == 0 && threadIdx.x == 0 && sdec_out != scale_src) *sdec_out = s_dec;
-
-  const int lane = threadIdx.x & 31;
-  const int g0 = lane & ~7;
-  const int64_t chunks_per_row = K >> 3;
-  const int64_t warp = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
-  for (int64_t base = warp * 32 * kUnroll; base < n_chunks; base += nwarps * 32 * kUnroll) {
-    uint4 v[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int64_t c = base + u * 32 + lane;
-      v[u] = (c < n_chunks) ? __ldg(x + c) : make_uint4(0u, 0u, 0u, 0u);
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int64_t c = base + u * 32 + lane;
-      // block amax over the lane pair holding the 16-element block
-      uint32_t mb = chunk_abs_max_bits(v[u]);
-      mb = max(mb, __shfl_xor_sync(0xFFFFFFFFu, mb, 1));
-      float r_b;
-      const uint32_t sb = nvfp4_block_scale(__uint_as_float(mb << 16), s_enc, &r_b);
-      float f[8];
-      unpack8(v[u], f);
-#pragma unroll
-      for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], r_b);
-      const uint32_t code = e2m1x8(f);
-      const uint32_t s0 = __shfl_sync(0xFFFFFFFFu, sb, g0);
-      const uint32_t s1 = __shfl_sync(0xFFFFFFFFu, sb, g0 + 2);
-      const uint32_t s2 = __shfl_sync(0xFFFFFFFFu, sb, g0 + 4);
-      const uint32_t s3 = __shfl_sync(0xFFFFFFFFu, sb, g0 + 6);
-      if (c < n_chunks) {
-        codes[c] = code;
-        if ((lane & 7) == 0) {
-          const int64_t row = c / chunks_per_row;
-          const int64_t col = (c - row * chunks_per_row) << 3;
-          *reinterpret_cast<uint32_t*>(scales + scale_offset(row, col >> 4, K)) =
-              s0 | (s1 << 8) | (s2 << 16) | (s3 << 24);
-        }
-      }
-    }
-  }
+  return s_dec;
 }
 
-// FP8 quantizer with one tensor scale (dynamic: S_dec = amax / 448).
+template <bool kDynamic, typename Idx>
+__global__ void __launch_bounds__(kThreads, kBlocksPerSm)
+    quant_nvfp4_kernel(const uint4* __restrict__ x, uint64_t n_chunks, int64_t K,
+                       const float* scale_src, float* sdec_out, uint32_t* __restrict__ codes,
+                       uint8_t* __restrict__ scales, unsigned* err, uint64_t timeout_ns) {
+  __shared__ float r_table[128];
+  Nvfp4Op<Idx> op;
+  op.r_table = r_table;
+  op.s_enc = encode_scale(tensor_scale<kDynamic>(scale_src, sdec_out, 2688.0f));
+  op.chunks_per_row = (Idx)(K >> 3);
+  op.K = K;
+  op.codes = codes;
+  op.scales = scales;
+  stream_tiles(x, n_chunks, op, err, timeout_ns);
+}
+
 template <bool kDynamic>
-__global__ void __launch_bounds__(kThreads) quant_fp8_kernel(const uint4* __restrict__ x,
-                                                             int64_t n_chunks,
-                                                             const float* scale_src,
-                                                             float* sdec_out,
-                                                             uint2* __restrict__ codes) {
-  float s_dec;
-  if (kDynamic) {
-    const float amax = *scale_src;
-    s_dec = (amax == 0.0f) ? 1.0f : __fdiv_rn(amax, 448.0f);
-  } else {
-    s_dec = *scale_src;
-  }
-  const float s_enc = encode_scale(s_dec);
-  if (blockIdx.x == 0 && threadIdx.x == 0 && sdec_out != scale_src) *sdec_out = s_dec;
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
-  for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < n_chunks; c += stride) {
-    float f[8];
-    unpack8(__ldg(x + c), f);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], s_enc);
-    codes[c] = make_uint2(e4m3x4(f[0], f[1], f[2], f[3]), e4m3x4(f[4], f[5], f[6], f[7]));
-  }
+__global__ void __launch_bounds__(kThreads, kBlocksPerSm)
+    quant_fp8_kernel(const uint4* __restrict__ x, uint64_t n_chunks, const float* scale_src,
+                     float* sdec_out, uint2* __restrict__ codes, unsigned* err,
+                     uint64_t timeout_ns) {
+  Fp8Op op;
+  op.s_enc = encode_scale(tensor_scale<kDynamic>(scale_src, sdec_out, 448.0f));
+  op.codes = codes;
+  stream_tiles(x, n_chunks, op, err, timeout_ns);
 }
 
 // FP8 weights, one scale per row: one warp per row, two passes over the row
-// (the second hits L1/L2).
+// (the second hits L1/L2).  Offline, once per layer.
 __global__ void __launch_bounds__(kThreads) quant_fp8_rows_kernel(const uint4* __restrict__ w,
                                                                   int64_t rows, int64_t K,
                                                                   float* __restrict__ s_rows,
@@ -179,56 +307,86 @@ __global__ void __launch_bounds__(kThreads) quant_fp8_rows_kernel(const uint4* _
   }
 }
 
-int grid_for(int64_t work_items, int items_per_block, int num_sms) {
-  const int64_t want = (work_items + items_per_block - 1) / items_per_block;
-  const int64_t cap = (int64_t)num_sms * (2048 / kThreads);
-  return (int)std::max<int64_t>(1, std::min(want, cap));
+// Opt each kernel into kSmem bytes of dynamic shared memory, once.
+template <auto kKern>
+cudaError_t set_smem() {
+  static const cudaError_t e =
+      cudaFuncSetAttribute(kKern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+  return e;
+}
+
+int stream_grid(uint64_t n_chunks, int num_sms) {
+  const uint64_t tiles = (n_chunks + kTileChunks - 1) / kTileChunks;
+  return (int)std::max<uint64_t>(1, std::min<uint64_t>(tiles, (uint64_t)num_sms * kBlocksPerSm));
 }
 
 }  // namespace
 
 cudaError_t launch_amax(const void* x, int64_t n_elems, unsigned* amax_bits, cudaStream_t s,
-                        int num_sms) {
+                        int num_sms, unsigned* err, uint64_t timeout_ns) {
   cudaError_t e = cudaMemsetAsync(amax_bits, 0, sizeof(unsigned), s);
   if (e != cudaSuccess) return e;
-  const int64_t n_chunks = n_elems / 8;
-  amax_bf16_kernel<<<grid_for(n_chunks, kThreads * kUnroll, num_sms), kThreads, 0, s>>>(
-      static_cast<const uint4*>(x), n_chunks, amax_bits);
+  if ((e = set_smem<amax_kernel>()) != cudaSuccess) return e;
+  const uint64_t n_chunks = (uint64_t)n_elems / 8;
+  amax_kernel<<<stream_grid(n_chunks, num_sms), kThreads, kSmem, s>>>(
+      static_cast<const uint4*>(x), n_chunks, amax_bits, err, timeout_ns);
+  return cudaGetLastError();
+}
+
+template <bool kDynamic>
+static cudaError_t launch_nvfp4_t(const void* x, int64_t M, int64_t K, const float* scale_src,
+                                  const qlin_nvfp4_t& out, cudaStream_t s, int num_sms,
+                                  unsigned* err, uint64_t timeout_ns) {
+  const uint64_t n_chunks = (uint64_t)M * (uint64_t)K / 8;
+  const int grid = stream_grid(n_chunks, num_sms);
+  auto* xin = static_cast<const uint4*>(x);
+  auto* codes = reinterpret_cast<uint32_t*>(out.codes);
+  cudaError_t e;
+  if (n_chunks < (1ull << 32)) {   // 32-bit index math is enough
+    auto kern = quant_nvfp4_kernel<kDynamic, uint32_t>;
+    if ((e = set_smem<quant_nvfp4_kernel<kDynamic, uint32_t>>()) != cudaSuccess) return e;
+    kern<<<grid, kThreads, kSmem, s>>>(xin, n_chunks, K, scale_src, out.tensor_scale, codes,
+                                      out.scales, err, timeout_ns);
+  } else {
+    auto kern = quant_nvfp4_kernel<kDynamic, uint64_t>;
+    if ((e = set_smem<quant_nvfp4_kernel<kDynamic, uint64_t>>()) != cudaSuccess) return e;
+    kern<<<grid, kThreads, kSmem, s>>>(xin, n_chunks, K, scale_src, out.tensor_scale, codes,
+                                      out.scales, err, timeout_ns);
+  }
   return cudaGetLastError();
 }
 
 cudaError_t launch_quant_nvfp4(const void* x, int64_t M, int64_t K, const float* scale_src,
                                bool dynamic, const qlin_nvfp4_t& out, cudaStream_t s,
-                               int num_sms) {
-  const int64_t n_chunks = M * K / 8;
-  const int grid = grid_for(n_chunks, kThreads * kUnroll, num_sms);
-  auto* xin = static_cast<const uint4*>(x);
-  auto* codes = reinterpret_cast<uint32_t*>(out.codes);
-  if (dynamic)
-    quant_nvfp4_kernel<true><<<grid, kThreads, 0, s>>>(xin, n_chunks, K, scale_src,
-                                                        out.tensor_scale, codes, out.scales);
-  else
-    quant_nvfp4_kernel<false><<<grid, kThreads, 0, s>>>(xin, n_chunks, K, scale_src,
-                                                         out.tensor_scale, codes, out.scales);
-  return cudaGetLastError();
+                               int num_sms, unsigned* err, uint64_t timeout_ns) {
+  return dynamic ? launch_nvfp4_t<true>(x, M, K, scale_src, out, s, num_sms, err, timeout_ns)
+                 : launch_nvfp4_t<false>(x, M, K, scale_src, out, s, num_sms, err, timeout_ns);
 }
 
 cudaError_t launch_quant_fp8(const void* x, int64_t M, int64_t K, const float* scale_src,
-                             bool dynamic, const qlin_fp8_t& out, cudaStream_t s, int num_sms) {
-  const int64_t n_chunks = M * K / 8;
-  const int grid = grid_for(n_chunks, kThreads * kUnroll, num_sms);
+                             bool dynamic, const qlin_fp8_t& out, cudaStream_t s, int num_sms,
+                             unsigned* err, uint64_t timeout_ns) {
+  const uint64_t n_chunks = (uint64_t)M * (uint64_t)K / 8;
+  const int grid = stream_grid(n_chunks, num_sms);
   auto* xin = static_cast<const uint4*>(x);
   auto* codes = reinterpret_cast<uint2*>(out.codes);
-  if (dynamic)
-    quant_fp8_kernel<true><<<grid, kThreads, 0, s>>>(xin, n_chunks, scale_src, out.scale, codes);
-  else
-    quant_fp8_kernel<false><<<grid, kThreads, 0, s>>>(xin, n_chunks, scale_src, out.scale, codes);
+  cudaError_t e;
+  if (dynamic) {
+    if ((e = set_smem<quant_fp8_kernel<true>>()) != cudaSuccess) return e;
+    quant_fp8_kernel<true><<<grid, kThreads, kSmem, s>>>(xin, n_chunks, scale_src, out.scale,
+                                                         codes, err, timeout_ns);
+  } else {
+    if ((e = set_smem<quant_fp8_kernel<false>>()) != cudaSuccess) return e;
+    quant_fp8_kernel<false><<<grid, kThreads, kSmem, s>>>(xin, n_chunks, scale_src, out.scale,
+                                                          codes, err, timeout_ns);
+  }
   return cudaGetLastError();
 }
 
 cudaError_t launch_quant_fp8_rows(const void* w, int64_t N, int64_t K, const qlin_fp8_t& out,
                                   cudaStream_t s, int num_sms) {
-  const int grid = grid_for(N, kThreads / 32, num_sms);
+  const int64_t want = (N + kThreads / 32 - 1) / (kThreads / 32);
+  const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)num_sms * 8));
   quant_fp8_rows_kernel<<<grid, kThreads, 0, s>>>(static_cast<const uint4*>(w), N, K, out.scale,
                                                   reinterpret_cast<uint2*>(out.codes));
   return cudaGetLastError();
