@@ -4,22 +4,26 @@
 // fused epilogue that writes the bf16 output and, optionally, re-quantizes it
 // to NVFP4 for the next layer.
 //
-// Kernel structure (one persistent CTA per SM, 320 threads):
-//   warp 0      TMA producer: A/W code tiles (tensor maps, 128-byte swizzle)
-//               and, for NVFP4, the 512-byte scale atoms (bulk copies) into a
-//               ring of shared-memory stages.
-//   warp 1      TMEM allocator and MMA issuer: per 32 bytes of K one
-//               tcgen05.mma (NVFP4: kind::mxf4nvf4 with scale_vec::4X, K = 64;
-//               FP8: kind::f8f6f4, K = 32) into an fp32 TMEM accumulator of
-//               128 lanes x BN columns.  NVFP4 scales are first moved
-//               shared -> TMEM with tcgen05.cp.
-//   warps 2-9   epilogue: tcgen05.ld of the accumulator (each warp its 32-lane
-//               quarter and one half of the columns), alpha scaling, bf16
-//               rounding, global stores, and the optional NVFP4 re-quantization
-//               of the bf16 values (one row per thread, so block amax is
-//               thread-local).
-// Tiles are 128 x BN output blocks, scheduled m-fastest so consecutive CTAs
-// share a weight tile in L2.  Every wait is bounded (see WaitCtl).
+// Two tile configurations share one kernel template:
+//   pair   256 x 256 output tiles on a CTA pair (a cluster of two CTAs on two
+//          SMs): one tcgen05 MMA of M = 256 (cta_group::2) issued by CTA 0
+//          drives both SMs' tensor cores; each CTA holds its own 128 rows of A
+//          and its own half of the W tile in shared memory.
+//   single 128 x 128 tiles on one CTA, for small M (the translator's linears).
+// Roles (12 warps, one persistent CTA per SM):
+//   warp 0      TMA producer: per pipeline stage one 4-D tensor copy per lane
+//               (A tile, W tile, A scale atoms, W scale atoms), issued by four
+//               lanes as a single instruction.  In a pair, CTA 1's copies
+//               complete on CTA 0's barriers (cta_group::2 form).
+//   warp 1      TMEM allocation; MMA issue (per 32 bytes of K one tcgen05.mma:
+//               NVFP4 kind::mxf4nvf4 scale_vec::4X with K = 64, FP8
+//               kind::f8f6f4 with K = 32) into an fp32 TMEM accumulator.
+//   warps 2-3   NVFP4: block scales shared -> TMEM (tcgen05.cp), beside the
+//               MMA stream.
+//   warps 4-11  epilogue: tcgen05.ld of the accumulator, alpha, bf16, TMA
+//               stores through swizzled staging, optional NVFP4 re-quantization
+//               of the bf16 values (one row per thread).
+// Every wait is bounded (see WaitCtl).
 #include <cstring>
 #include <mutex>
 
@@ -36,6 +40,10 @@ constexpr int kEpiWarps = 8;
 constexpr int kEpiWarp0 = 4;   // warps 0-3: producer, MMA, two scale-copy warps
 constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
 constexpr int kSmemBudget = 232448 - 2048;  // opt-in shared memory minus barriers/alignment
+#ifndef QLIN_TMA_SPLIT
+#define QLIN_TMA_SPLIT 1
+#endif
+constexpr int kSplit = QLIN_TMA_SPLIT;      // row boxes per operand tile and stage
 
 constexpr int pow2_at_least(int x) {
   int p = 32;
@@ -43,11 +51,13 @@ constexpr int pow2_at_least(int x) {
   return p;
 }
 
-template <bool kFp4, int kBN>
+// kPair: a CTA pair runs one tcgen05 MMA of M = 256 (cta_group::2); each CTA
+// holds its own 128 rows of A and its own half of the W tile.
+template <bool kFp4, int kBN, bool kPair = false>
 struct Cfg {
   static constexpr int kSfbAtoms = kFp4 ? (kBN + 127) / 128 : 0;
   static constexpr int kABytes = kBM * kRowBytes;
-  static constexpr int kBBytes = kBN * kRowBytes;
+  static constexpr int kBBytes = (kPair ? kBN / 2 : kBN) * kRowBytes;
   static constexpr int kSfaBytes = kFp4 ? kStepsPerStage * 512 : 0;
   static constexpr int kSfbBytes = kFp4 ? kSfbAtoms * kStepsPerStage * 512 : 0;
   static constexpr int kStageBytes = kABytes + kBBytes + kSfaBytes + kSfbBytes;
@@ -106,16 +116,15 @@ __device__ __forceinline__ void st_global_v4(void* p, uint32_t a, uint32_t b, ui
                : "memory");
 }
 
-template <bool kFp4, int kBN, int kCM, bool kRequant>
+template <bool kFp4, int kBN, bool kPair, bool kRequant>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_a,
                 const __grid_constant__ CUtensorMap tmap_b,
+                const __grid_constant__ CUtensorMap tmap_sfa,
+                const __grid_constant__ CUtensorMap tmap_sfb,
                 const __grid_constant__ CUtensorMap tmap_y, const KParams p) {
-  using C = Cfg<kFp4, kBN>;
-  // kCM CTAs of a cluster take kCM consecutive M tiles of the same N tile;
-  // each loads 1/kCM of the weight tile (and of its scales) and multicasts
-  // it to all, so W is read from L2 once per cluster.
-  constexpr int kBRows = kBN / kCM;
+  using C = Cfg<kFp4, kBN, kPair>;
+  constexpr int kCM = kPair ? 2 : 1;          // CTAs per cluster (M tiles per cluster tile)
   constexpr uint16_t kMask = (uint16_t)((1u << kCM) - 1u);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -134,18 +143,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int rank = kCM > 1 ? (int)cluster_ctarank() : 0;
+  const int rank = kPair ? (int)cluster_ctarank() : 0;
+  const bool leader = rank == 0;   // a pair's MMA / scale-copy CTA
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], kCM);   // one arrival from the MMA warp of each CTA
+      mbar_init(&empty[s], 1);
       mbar_init(&sf_ready[s], 2);   // one commit per scale-copy warp
       mbar_init(&sf_full[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tmem_full[a], 1);
-      mbar_init(&tmem_empty[a], kEpiWarps);
+      mbar_init(&tmem_empty[a], kCM * kEpiWarps);   // every epilogue warp of the cluster
     }
     mbar_init(mma_done, 1);
     mbar_init(&sf_done[0], 1);
@@ -153,14 +163,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     *abort_flag = 0;
     mbar_fence_init();
   }
-  if (warp == 0 && lane == 0) {
-    prefetch_tmap(&tmap_a);
-    prefetch_tmap(&tmap_b);
+  if (warp == 0 && lane < (kFp4 ? 4 : 2))
+    prefetch_tmap(lane == 0 ? &tmap_a : lane == 1 ? &tmap_b : lane == 2 ? &tmap_sfa : &tmap_sfb);
+  if (warp == 1) {
+    if (kPair)
+      tmem_alloc_pair(tmem_slot, C::kTmemCols);
+    else
+      tmem_alloc(tmem_slot, C::kTmemCols);
   }
-  if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
   tc_fence_before();
-  if (kCM > 1)
-    cluster_sync();   // peers' barriers exist before any multicast reaches them
+  if (kPair)
+    cluster_sync();   // the peer's barriers exist before any copy completes on them
   else
     __syncthreads();
   tc_fence_after();
@@ -176,25 +189,36 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int64_t k_bytes = kFp4 ? p.K / 2 : p.K;
   const int num_kb = (int)((k_bytes + kRowBytes - 1) / kRowBytes);
   const int k_steps = (int)(k_bytes / 32);
-  const int64_t k_atoms = p.K / 64;  // 4-scale atom columns (NVFP4)
 
   if (warp == 0) {
     // ------------------------------------------------------ TMA producer ---
-    // A TMA instruction occupies its issuing thread for hundreds of cycles,
-    // so the stage's copies are issued by several lanes executing the SAME
-    // instruction with per-lane operands: lanes 0 and 1 one tensor load (A
-    // tile, W tile), lanes 2.. one bulk copy (A scales, W scale rows).
-    const int nlanes = kFp4 ? 3 + C::kSfbAtoms : 2;
+    // One 4-D tensor copy per lane (0: A tile, 1: W tile, 2: A scale atoms,
+    // 3: W scale atoms), all four issued as ONE instruction: a TMA copy holds
+    // its issuing thread for hundreds of cycles, so issuing them one by one
+    // would starve the tensor cores.  Out-of-range boxes (rows past M or N, K
+    // atoms past the end) are zero-filled and still count their full bytes,
+    // so every stage expects the same byte counts.
+    // Each operand tile is split into kSplit row boxes, one lane each, so
+    // more copies run at once (lanes [0, kSplit): A parts, [kSplit, 2 kSplit):
+    // W parts, then A scales, W scales).
+    constexpr int kOpLanes = 2 * kSplit;
+    const int nlanes = kFp4 ? kOpLanes + 2 : kOpLanes;
     if (lane < nlanes) {
+      const bool is_scale = lane >= kOpLanes;
+      const int part = lane % kSplit;
+      const CUtensorMap* map = lane < kSplit      ? &tmap_a
+                               : lane < kOpLanes  ? &tmap_b
+                               : lane == kOpLanes ? &tmap_sfa
+                                                  : &tmap_sfb;
+      uint64_t* bars = is_scale ? sf_full : full;
+      // barrier each copy completes on: this CTA's, or in a pair CTA 0's
+      const uint32_t bar0 = kPair ? mapa_shared(bars, 0) : smem_u32(bars);
       int stage = 0;
       uint32_t phase = 0;
       int issued = 0;
-      const int n_atom_rows = (int)((p.N + 127) / 128);
-      const uint16_t self_mask = (uint16_t)(1u << rank);
       for (int ct = cid; ct < num_ctiles; ct += ncl) {
         const int nb = ct / groups_m;
         const int mb = (ct % groups_m) * kCM + rank;
-        const bool m_live = mb < tiles_m;   // the last group may be partly past M
         bool ok = true;
         for (int kb = 0; kb < num_kb; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, ctl)) {
@@ -203,43 +227,32 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           uint8_t* sA = smem + stage * C::kStageBytes;
           uint8_t* sB = sA + C::kABytes;
-          const int nat = min(kStepsPerStage, k_steps - kb * kStepsPerStage);
-          const int nsfb = kFp4 ? min(C::kSfbAtoms, n_atom_rows - nb * (kBN / 128)) : 0;
-          if (lane == 0) mbar_arrive_expect_tx(&full[stage], C::kABytes + C::kBBytes);
-          if (kFp4 && lane == 2)   // the scales complete on their own barrier
-            mbar_arrive_expect_tx(&sf_full[stage],
-                                  (uint32_t)(nat * 512 * ((m_live ? 1 : 0) + nsfb)));
+          if (leader && lane == 0)
+            mbar_arrive_expect_tx(&full[stage], kCM * (C::kABytes + C::kBBytes));
+          if (kFp4 && leader && lane == kOpLanes)
+            mbar_arrive_expect_tx(&sf_full[stage], kCM * (C::kSfaBytes + C::kSfbBytes));
           __syncwarp((1u << nlanes) - 1u);
-          // operand tiles
-          if (lane < 2) {
-            const bool is_a = lane == 0;
-            const CUtensorMap* map = is_a ? &tmap_a : &tmap_b;
-            const int32_t y = is_a ? mb * kBM : nb * kBN + rank * kBRows;
-            uint8_t* dst = is_a ? sA : sB + rank * kBRows * kRowBytes;
-            if (kCM == 1)
-              tma_load_2d(dst, map, &full[stage], kb * kRowBytes, y);
-            else
-              tma_load_2d_mc(dst, map, &full[stage], kb * kRowBytes, y,
-                             is_a ? self_mask : kMask);
-          } else if (kFp4) {
-            // block scales: lane 2 the A atoms, lane 3 + r the W atom row r
-            const bool is_a = lane == 2;
-            const int r = lane - 3;
-            const bool live = is_a ? m_live : (r < nsfb && r % kCM == rank);
-            const uint8_t* src =
-                is_a ? p.sfa + ((int64_t)mb * k_atoms + kb * kStepsPerStage) * 512
-                     : p.sfb + ((int64_t)(nb * (kBN / 128) + r) * k_atoms + kb * kStepsPerStage) *
-                                   512;
-            uint8_t* dst = is_a ? sB + C::kBBytes
-                                : sB + C::kBBytes + C::kSfaBytes + r * kStepsPerStage * 512;
-            if (live) {
-              if (kCM == 1)
-                bulk_load(dst, src, (uint32_t)nat * 512, &sf_full[stage]);
-              else
-                bulk_load_mc(dst, src, (uint32_t)nat * 512, &sf_full[stage],
-                             is_a ? self_mask : kMask);
-            }
+          uint8_t* dst;
+          int32_t c0, c1, c2, c3;
+          constexpr int kARows = kBM / kSplit, kBRowsPart = kBN / kCM / kSplit;
+          if (lane < kSplit) {              // A: part of this CTA's M tile
+            dst = sA + part * kARows * kRowBytes;
+            c0 = kb * kRowBytes; c1 = mb * kBM + part * kARows; c2 = 0; c3 = 0;
+          } else if (lane < kOpLanes) {     // W: part of this CTA's rows of the N tile
+            dst = sB + part * kBRowsPart * kRowBytes;
+            c0 = kb * kRowBytes; c1 = nb * kBN + rank * (kBN / kCM) + part * kBRowsPart;
+            c2 = 0; c3 = 0;
+          } else if (lane == kOpLanes) {    // A scale atoms of this stage
+            dst = sB + C::kBBytes; c0 = 0; c1 = 0; c2 = kb * kStepsPerStage; c3 = mb;
+          } else {                          // W scale atoms (all atom rows of the N tile)
+            dst = sB + C::kBBytes + C::kSfaBytes; c0 = 0; c1 = 0; c2 = kb * kStepsPerStage;
+            c3 = nb * C::kSfbAtoms;
           }
+          const uint32_t bar = bar0 + (uint32_t)(stage * 8);
+          if (kPair)
+            tma_load_4d_pair(dst, map, bar, c0, c1, c2, c3);
+          else
+            tma_load_4d(dst, map, bar, c0, c1, c2, c3);
           ++issued;
           if (++stage == C::kStages) {
             stage = 0;
@@ -248,10 +261,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!ok) break;
       }
-      // Wait for the last copies into this CTA (normally complete long ago)
-      // so none is in flight when the CTA exits.
-      if (lane == 0 || (kFp4 && lane == 2)) {
-        uint64_t* bars = lane == 0 ? full : sf_full;
+      // Let the last copies into this CTA land before it exits (the barriers
+      // that count them live in CTA 0; its producer drains them).
+      if (leader && (lane == 0 || (kFp4 && lane == kOpLanes))) {
         const int n_drain = min(issued, C::kStages);
         for (int i = 0; i < n_drain; ++i) {
           if (--stage < 0) {
@@ -264,8 +276,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     // ------------------------------------------------------- MMA issuer ---
-    if (lane == 0) {
-      const uint32_t idesc = kFp4 ? idesc_nvfp4(kBN) : idesc_fp8(kBN);
+    if (lane == 0 && leader) {
+      constexpr int kMmaM = kPair ? 256 : 128;
+      const uint32_t idesc = kFp4 ? idesc_nvfp4(kBN, kMmaM) : idesc_fp8(kBN, kMmaM);
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
@@ -293,24 +306,32 @@ __global__ void __launch_bounds__(kThreads, 1)
               const uint32_t sfa_t = tmem_base + (uint32_t)(C::kSfColBase +
                                                             (stage * kStepsPerStage + j) *
                                                                 C::kSfColsPerStep);
-              mma_nvfp4(d_tmem, adesc, bdesc, idesc, sfa_t, sfa_t + 4, accumulate);
+              if (kPair)
+                mma_nvfp4_pair(d_tmem, adesc, bdesc, idesc, sfa_t, sfa_t + 4, accumulate);
+              else
+                mma_nvfp4(d_tmem, adesc, bdesc, idesc, sfa_t, sfa_t + 4, accumulate);
             } else {
-              mma_fp8(d_tmem, adesc, bdesc, idesc, accumulate);
+              if (kPair)
+                mma_fp8_pair(d_tmem, adesc, bdesc, idesc, accumulate);
+              else
+                mma_fp8(d_tmem, adesc, bdesc, idesc, accumulate);
             }
           }
-          // the stage is free once this CTA's MMAs have read it: tell every
-          // CTA of the cluster (their producers multicast into it)
-          if (kCM == 1)
-            tc_commit(&empty[stage]);
+          // the stage is free once the MMAs have read it (both CTAs' halves)
+          if (kPair)
+            tc_commit_pair_mc(&empty[stage], kMask);
           else
-            tc_commit_mc(&empty[stage], kMask);
+            tc_commit(&empty[stage]);
           if (++stage == C::kStages) {
             stage = 0;
             phase ^= 1u;
           }
         }
         if (!ok) break;
-        tc_commit(&tmem_full[acc]);
+        if (kPair)
+          tc_commit_pair_mc(&tmem_full[acc], kMask);   // both CTAs' epilogues
+        else
+          tc_commit(&tmem_full[acc]);
         if (C::kNumAcc == 2) {
           acc ^= 1;
           if (acc == 0) acc_phase ^= 1u;
@@ -319,15 +340,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       // Every MMA / scale copy issued must finish before TMEM is released.
-      tc_commit(mma_done);
+      if (kPair)
+        tc_commit_pair_mc(mma_done, 1);
+      else
+        tc_commit(mma_done);
       mbar_drain(mma_done, 0, p.timeout_ns, p.err);
     }
   } else if (warp == 2 || warp == 3) {
     // --------------------------------------------- NVFP4 scale copies ---
     // Block scales move shared -> TMEM from two threads of their own (a
     // tcgen05.cp occupies its issuing thread ~50 cycles), beside the MMA
-    // stream: warp 2 the A atoms and W atom row 0, warp 3 W atom row 1.
-    if (kFp4 && lane == 0) {
+    // stream: warp 2 the A atoms and W atom row 0, warp 3 W atom row 1.  In a
+    // pair, CTA 0's copies fill both SMs' TMEM from their own shared memory.
+    if (kFp4 && lane == 0 && leader) {
       const int sw = warp - 2;
       int stage = 0;
       uint32_t phase = 0;
@@ -347,13 +372,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                           (stage * kStepsPerStage + j) *
                                                               C::kSfColsPerStep);
             if (sw == 0) {
-              tc_cp_scales(sfa_t, sdesc_scales(sSFA + j * 512));
-              tc_cp_scales(sfa_t + 4, sdesc_scales(sSFB + j * 512));
+              if (kPair) {
+                tc_cp_scales_pair(sfa_t, sdesc_scales(sSFA + j * 512));
+                tc_cp_scales_pair(sfa_t + 4, sdesc_scales(sSFB + j * 512));
+              } else {
+                tc_cp_scales(sfa_t, sdesc_scales(sSFA + j * 512));
+                tc_cp_scales(sfa_t + 4, sdesc_scales(sSFB + j * 512));
+              }
             } else if (C::kSfbAtoms > 1) {
-              tc_cp_scales(sfa_t + 8, sdesc_scales(sSFB + kStepsPerStage * 512 + j * 512));
+              if (kPair)
+                tc_cp_scales_pair(sfa_t + 8,
+                                  sdesc_scales(sSFB + kStepsPerStage * 512 + j * 512));
+              else
+                tc_cp_scales(sfa_t + 8, sdesc_scales(sSFB + kStepsPerStage * 512 + j * 512));
             }
           }
-          tc_commit(&sf_ready[stage]);
+          if (kPair)
+            tc_commit_pair_mc(&sf_ready[stage], 1);
+          else
+            tc_commit(&sf_ready[stage]);
           if (++stage == C::kStages) {
             stage = 0;
             phase ^= 1u;
@@ -361,7 +398,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!ok) break;
       }
-      tc_commit(&sf_done[sw]);
+      if (kPair)
+        tc_commit_pair_mc(&sf_done[sw], 1);
+      else
+        tc_commit(&sf_done[sw]);
       mbar_drain(&sf_done[sw], 0, p.timeout_ns, p.err);
     }
   } else {
@@ -435,7 +475,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       // The accumulator is in registers: hand it back to the MMA warp.
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tmem_empty[acc]);
+      if (lane == 0) {
+        if (kPair && rank == 1)
+          mbar_arrive_cluster(mapa_shared(&tmem_empty[acc], 0));   // CTA 0 owns the MMA
+        else
+          mbar_arrive(&tmem_empty[acc]);
+      }
       if (C::kNumAcc == 2) {
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1u;
@@ -509,13 +554,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   // No CTA of the cluster may exit while a peer can still multicast into it
   // or arrive on its barriers.
   tc_fence_before();
-  if (kCM > 1)
+  if (kPair)
     cluster_sync();
   else
     __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, C::kTmemCols);
+    if (kPair)
+      tmem_dealloc_pair(tmem_base, C::kTmemCols);
+    else
+      tmem_dealloc(tmem_base, C::kTmemCols);
   }
 }
 
@@ -555,17 +603,55 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-template <bool kFp4, int kBN, int kCM, bool kRequant>
+// 4-D uint8 tensor map (dims innermost first, strides in bytes for dims 1-3).
+CUresult encode_u8_4d(CUtensorMap* map, const void* base, const cuuint64_t (&dims)[4],
+                      const cuuint64_t (&strides)[3], const cuuint32_t (&box)[4],
+                      CUtensorMapSwizzle swz) {
+  EncodeTiledFn fn = encode_fn();
+  if (fn == nullptr) return CUDA_ERROR_NOT_FOUND;
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+// Codes [rows, k_bytes] as a 4-D tensor with two unit dimensions, 128-byte x
+// box_rows boxes with the 128-byte swizzle.
+CUresult encode_codes(CUtensorMap* map, const void* base, uint64_t k_bytes, uint64_t rows,
+                      uint32_t box_rows) {
+  const cuuint64_t dims[4] = {k_bytes, rows, 1, 1};
+  const cuuint64_t strides[3] = {k_bytes, k_bytes * rows, k_bytes * rows};
+  const cuuint32_t box[4] = {kRowBytes, box_rows, 1, 1};
+  return encode_u8_4d(map, base, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+// Swizzled block scales as {16 B, 32 atom rows, K/64 atoms, row blocks}: a box
+// of {16, 32, 4, n} is n row blocks' four atoms of one pipeline stage, laid
+// out in shared memory exactly as in global memory.
+CUresult encode_scales(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K,
+                       uint32_t row_blocks_per_box) {
+  const cuuint64_t atoms = K / 64;
+  const cuuint64_t dims[4] = {16, 32, atoms, (rows + 127) / 128};
+  const cuuint64_t strides[3] = {16, 512, atoms * 512};
+  const cuuint32_t box[4] = {16, 32, (cuuint32_t)kStepsPerStage, row_blocks_per_box};
+  return encode_u8_4d(map, base, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE);
+}
+
+template <bool kFp4, int kBN, bool kPair, bool kRequant>
 cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned* err,
                        uint64_t timeout_ns) {
-  using C = Cfg<kFp4, kBN>;
+  using C = Cfg<kFp4, kBN, kPair>;
+  constexpr int kCM = kPair ? 2 : 1;
   const uint64_t k_bytes = kFp4 ? (uint64_t)a.K / 2 : (uint64_t)a.K;
-  CUtensorMap ta, tb, ty;
+  CUtensorMap ta, tb, tsa, tsb, ty;
+  std::memset(&tsa, 0, sizeof tsa);
+  std::memset(&tsb, 0, sizeof tsb);
   std::memset(&ty, 0, sizeof ty);
-  if (encode_tensor_map_2d_u8(&ta, a.a_codes, k_bytes, (uint64_t)a.M, kRowBytes, kBM) !=
-          CUDA_SUCCESS ||
-      encode_tensor_map_2d_u8(&tb, a.w_codes, k_bytes, (uint64_t)a.N, kRowBytes, kBN / kCM) !=
-          CUDA_SUCCESS ||
+  if (encode_codes(&ta, a.a_codes, k_bytes, (uint64_t)a.M, kBM / kSplit) != CUDA_SUCCESS ||
+      encode_codes(&tb, a.w_codes, k_bytes, (uint64_t)a.N, kBN / kCM / kSplit) != CUDA_SUCCESS ||
+      (kFp4 && (encode_scales(&tsa, a.sfa, (uint64_t)a.M, (uint64_t)a.K, 1) != CUDA_SUCCESS ||
+                encode_scales(&tsb, a.sfb, (uint64_t)a.N, (uint64_t)a.K, C::kSfbAtoms) !=
+                    CUDA_SUCCESS)) ||
       (a.y != nullptr && encode_tensor_map_out_bf16(&ty, a.y, (uint64_t)a.N, (uint64_t)a.M) !=
                              CUDA_SUCCESS))
     return cudaErrorInvalidValue;
@@ -587,7 +673,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   p.rq_cols = a.rq_cols;
   p.err = err;
   p.timeout_ns = timeout_ns;
-  auto kern = gemm_kernel<kFp4, kBN, kCM, kRequant>;
+  auto kern = gemm_kernel<kFp4, kBN, kPair, kRequant>;
 
   cudaLaunchConfig_t cfg{};
   cudaLaunchAttribute attr[1];
@@ -619,23 +705,23 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   const int64_t ctiles = ((tiles_m + kCM - 1) / kCM) * ((a.N + kBN - 1) / kBN);
   const int clusters = (int)std::min<int64_t>(ctiles, std::min(max_clusters, num_sms / kCM));
   cfg.gridDim = dim3((unsigned)(clusters * kCM), 1, 1);
-  return cudaLaunchKernelEx(&cfg, kern, ta, tb, ty, p);
+  return cudaLaunchKernelEx(&cfg, kern, ta, tb, tsa, tsb, ty, p);
 }
 
 template <bool kFp4>
 cudaError_t dispatch_bn(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned* err,
                         uint64_t timeout_ns) {
-  // 128 x 256 tiles in clusters of two along M (shared weight tile) when they
-  // fill the machine, else 128 x 128 single-CTA tiles (small M).
+  // 256 x 256 tiles on CTA pairs when they fill the machine, else 128 x 128
+  // single-CTA tiles (small M).
   const int64_t tiles256 = ((a.M + kBM - 1) / kBM) * ((a.N + 255) / 256);
   const bool wide = tiles256 >= num_sms;
   if constexpr (kFp4) {
     if (a.next_scale != nullptr)
-      return wide ? launch_cfg<true, 256, 2, true>(a, s, num_sms, err, timeout_ns)
-                  : launch_cfg<true, 128, 1, true>(a, s, num_sms, err, timeout_ns);
+      return wide ? launch_cfg<true, 256, true, true>(a, s, num_sms, err, timeout_ns)
+                  : launch_cfg<true, 128, false, true>(a, s, num_sms, err, timeout_ns);
   }
-  return wide ? launch_cfg<kFp4, 256, 2, false>(a, s, num_sms, err, timeout_ns)
-              : launch_cfg<kFp4, 128, 1, false>(a, s, num_sms, err, timeout_ns);
+  return wide ? launch_cfg<kFp4, 256, true, false>(a, s, num_sms, err, timeout_ns)
+              : launch_cfg<kFp4, 128, false, false>(a, s, num_sms, err, timeout_ns);
 }
 
 }  // namespace
