@@ -38,7 +38,14 @@ constexpr int kRowBytes = 128;      // bytes of K per stage and row: one swizzle
 constexpr int kStepsPerStage = 4;   // one MMA per 32 bytes of K
 constexpr int kEpiWarps = 8;
 constexpr int kEpiWarp0 = 4;   // warps 0-3: producer, MMA, two scale-copy warps
-constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
+#ifndef QLIN_PRODUCERS
+#define QLIN_PRODUCERS 1
+#endif
+// TMA producer warps: warp 0, then extra warps after the epilogue warps.  A
+// TMA tensor copy holds its issuing warp for hundreds of cycles, so several
+// warps take turns over the pipeline stages.
+constexpr int kProducers = QLIN_PRODUCERS;
+constexpr int kThreads = (kEpiWarp0 + kEpiWarps + kProducers - 1) * 32;
 constexpr int kSmemBudget = 232448 - 2048;  // opt-in shared memory minus barriers/alignment
 #ifndef QLIN_TMA_SPLIT
 #define QLIN_TMA_SPLIT 1
@@ -190,7 +197,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int num_kb = (int)((k_bytes + kRowBytes - 1) / kRowBytes);
   const int k_steps = (int)(k_bytes / 32);
 
-  if (warp == 0) {
+  const int producer = warp == 0 ? 0 : warp - (kEpiWarp0 + kEpiWarps) + 1;
+  if (warp == 0 || warp >= kEpiWarp0 + kEpiWarps) {
     // ------------------------------------------------------ TMA producer ---
     // One 4-D tensor copy per lane (0: A tile, 1: W tile, 2: A scale atoms,
     // 3: W scale atoms), all four issued as ONE instruction: a TMA copy holds
@@ -215,12 +223,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t bar0 = kPair ? mapa_shared(bars, 0) : smem_u32(bars);
       int stage = 0;
       uint32_t phase = 0;
-      int issued = 0;
+      int issued = 0;     // stages of this CTA's sequence, whichever warp issued them
       for (int ct = cid; ct < num_ctiles; ct += ncl) {
         const int nb = ct / groups_m;
         const int mb = (ct % groups_m) * kCM + rank;
         bool ok = true;
         for (int kb = 0; kb < num_kb; ++kb) {
+          if (kProducers > 1 && issued % kProducers != producer) {   // another warp's stage
+            ++issued;
+            if (++stage == C::kStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+            continue;
+          }
           if (!mbar_wait(&empty[stage], phase ^ 1u, ctl)) {
             ok = false;
             break;
@@ -243,10 +259,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             c0 = kb * kRowBytes; c1 = nb * kBN + rank * (kBN / kCM) + part * kBRowsPart;
             c2 = 0; c3 = 0;
           } else if (lane == kOpLanes) {    // A scale atoms of this stage
-            dst = sB + C::kBBytes; c0 = 0; c1 = 0; c2 = kb * kStepsPerStage; c3 = mb;
+            dst = sB + C::kBBytes; c0 = kb * kStepsPerStage * 64; c1 = mb; c2 = 0; c3 = 0;
           } else {                          // W scale atoms (all atom rows of the N tile)
-            dst = sB + C::kBBytes + C::kSfaBytes; c0 = 0; c1 = 0; c2 = kb * kStepsPerStage;
-            c3 = nb * C::kSfbAtoms;
+            dst = sB + C::kBBytes + C::kSfaBytes; c0 = kb * kStepsPerStage * 64;
+            c1 = nb * C::kSfbAtoms; c2 = 0; c3 = 0;
           }
           const uint32_t bar = bar0 + (uint32_t)(stage * 8);
           if (kPair)
@@ -263,7 +279,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // Let the last copies into this CTA land before it exits (the barriers
       // that count them live in CTA 0; its producer drains them).
-      if (leader && (lane == 0 || (kFp4 && lane == kOpLanes))) {
+      if (leader && producer == 0 && (lane == 0 || (kFp4 && lane == kOpLanes))) {
         const int n_drain = min(issued, C::kStages);
         for (int i = 0; i < n_drain; ++i) {
           if (--stage < 0) {
@@ -603,15 +619,16 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 4-D uint8 tensor map (dims innermost first, strides in bytes for dims 1-3).
-CUresult encode_u8_4d(CUtensorMap* map, const void* base, const cuuint64_t (&dims)[4],
-                      const cuuint64_t (&strides)[3], const cuuint32_t (&box)[4],
-                      CUtensorMapSwizzle swz) {
+// 4-D tensor map (dims innermost first, in elements; strides in bytes for
+// dims 1-3).
+CUresult encode_4d(CUtensorMap* map, CUtensorMapDataType type, const void* base,
+                   const cuuint64_t (&dims)[4], const cuuint64_t (&strides)[3],
+                   const cuuint32_t (&box)[4], CUtensorMapSwizzle swz) {
   EncodeTiledFn fn = encode_fn();
   if (fn == nullptr) return CUDA_ERROR_NOT_FOUND;
   const cuuint32_t estr[4] = {1, 1, 1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<void*>(base), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  return fn(map, type, 4, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
@@ -622,19 +639,23 @@ CUresult encode_codes(CUtensorMap* map, const void* base, uint64_t k_bytes, uint
   const cuuint64_t dims[4] = {k_bytes, rows, 1, 1};
   const cuuint64_t strides[3] = {k_bytes, k_bytes * rows, k_bytes * rows};
   const cuuint32_t box[4] = {kRowBytes, box_rows, 1, 1};
-  return encode_u8_4d(map, base, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B);
+  return encode_4d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base, dims, strides, box,
+                   CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
-// Swizzled block scales as {16 B, 32 atom rows, K/64 atoms, row blocks}: a box
-// of {16, 32, 4, n} is n row blocks' four atoms of one pipeline stage, laid
-// out in shared memory exactly as in global memory.
+// Swizzled block scales: the atoms of one 128-row block are contiguous along
+// K (512 bytes per 64 elements of K), so the scales are a [row blocks, K]
+// tensor of 8-byte words.  A box of {256 words, n row blocks} is the four
+// atoms of one pipeline stage for n row blocks (2 KB each, 16 rows of 128
+// bytes per request stream instead of 128 of 16 bytes), laid out in shared
+// memory exactly as in global memory.
 CUresult encode_scales(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K,
                        uint32_t row_blocks_per_box) {
-  const cuuint64_t atoms = K / 64;
-  const cuuint64_t dims[4] = {16, 32, atoms, (rows + 127) / 128};
-  const cuuint64_t strides[3] = {16, 512, atoms * 512};
-  const cuuint32_t box[4] = {16, 32, (cuuint32_t)kStepsPerStage, row_blocks_per_box};
-  return encode_u8_4d(map, base, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE);
+  const cuuint64_t dims[4] = {K, (rows + 127) / 128, 1, 1};
+  const cuuint64_t strides[3] = {K * 8, K * 8 * dims[1], K * 8 * dims[1]};
+  const cuuint32_t box[4] = {(cuuint32_t)(kStepsPerStage * 64), row_blocks_per_box, 1, 1};
+  return encode_4d(map, CU_TENSOR_MAP_DATA_TYPE_UINT64, base, dims, strides, box,
+                   CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
 template <bool kFp4, int kBN, bool kPair, bool kRequant>
