@@ -343,9 +343,13 @@ __device__ __forceinline__ uint32_t mapa_shared(const void* p, uint32_t rank) {
 }
 
 // Arrive on an mbarrier given by its shared::cluster address (any CTA of the
-// cluster), with release semantics at cluster scope.
+// cluster).  Release at the default (CTA) scope: the only thing published is
+// that this CTA's tcgen05.ld reads have completed (tcgen05.wait::ld plus
+// tcgen05.fence::before_thread_sync come first), not generic memory writes.
+// A cluster-scope release costs about a microsecond per arrival under TMA
+// load, which stalls the MMA issuer waiting on this barrier.
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
                : "memory");
 }
 

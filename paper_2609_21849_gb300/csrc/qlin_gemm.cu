@@ -38,14 +38,7 @@ constexpr int kRowBytes = 128;      // bytes of K per stage and row: one swizzle
 constexpr int kStepsPerStage = 4;   // one MMA per 32 bytes of K
 constexpr int kEpiWarps = 8;
 constexpr int kEpiWarp0 = 4;   // warps 0-3: producer, MMA, two scale-copy warps
-#ifndef QLIN_PRODUCERS
-#define QLIN_PRODUCERS 1
-#endif
-// TMA producer warps: warp 0, then extra warps after the epilogue warps.  A
-// TMA tensor copy holds its issuing warp for hundreds of cycles, so several
-// warps take turns over the pipeline stages.
-constexpr int kProducers = QLIN_PRODUCERS;
-constexpr int kThreads = (kEpiWarp0 + kEpiWarps + kProducers - 1) * 32;
+constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
 constexpr int kSmemBudget = 232448 - 2048;  // opt-in shared memory minus barriers/alignment
 #ifndef QLIN_TMA_SPLIT
 #define QLIN_TMA_SPLIT 1
@@ -197,8 +190,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int num_kb = (int)((k_bytes + kRowBytes - 1) / kRowBytes);
   const int k_steps = (int)(k_bytes / 32);
 
-  const int producer = warp == 0 ? 0 : warp - (kEpiWarp0 + kEpiWarps) + 1;
-  if (warp == 0 || warp >= kEpiWarp0 + kEpiWarps) {
+  if (warp == 0) {
     // ------------------------------------------------------ TMA producer ---
     // One 4-D tensor copy per lane (0: A tile, 1: W tile, 2: A scale atoms,
     // 3: W scale atoms), all four issued as ONE instruction: a TMA copy holds
@@ -223,20 +215,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t bar0 = kPair ? mapa_shared(bars, 0) : smem_u32(bars);
       int stage = 0;
       uint32_t phase = 0;
-      int issued = 0;     // stages of this CTA's sequence, whichever warp issued them
+      int issued = 0;
       for (int ct = cid; ct < num_ctiles; ct += ncl) {
         const int nb = ct / groups_m;
         const int mb = (ct % groups_m) * kCM + rank;
         bool ok = true;
         for (int kb = 0; kb < num_kb; ++kb) {
-          if (kProducers > 1 && issued % kProducers != producer) {   // another warp's stage
-            ++issued;
-            if (++stage == C::kStages) {
-              stage = 0;
-              phase ^= 1u;
-            }
-            continue;
-          }
           if (!mbar_wait(&empty[stage], phase ^ 1u, ctl)) {
             ok = false;
             break;
@@ -279,7 +263,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // Let the last copies into this CTA land before it exits (the barriers
       // that count them live in CTA 0; its producer drains them).
-      if (leader && producer == 0 && (lane == 0 || (kFp4 && lane == kOpLanes))) {
+      if (leader && (lane == 0 || (kFp4 && lane == kOpLanes))) {
         const int n_drain = min(issued, C::kStages);
         for (int i = 0; i < n_drain; ++i) {
           if (--stage < 0) {
