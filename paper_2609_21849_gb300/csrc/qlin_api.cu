@@ -117,6 +117,17 @@ qlin_status check_workspace(void* ws, size_t ws_bytes) {
   } while (0)
 
 }  // namespace
+// Dynamic NVFP4 activation quantization: one read of x when it fits on chip,
+// else the amax pass then the quantizer.  ws: at least two device words.
+cudaError_t quant_nvfp4_dynamic(const void* x, int64_t M, int64_t K, const qlin_nvfp4_t& out,
+                                unsigned* ws, cudaStream_t s, int sms, unsigned* status) {
+  cudaError_t e = launch_quant_nvfp4_onepass(x, M, K, out, ws, s, sms, status, timeout());
+  if (e != cudaErrorNotSupported) return e;
+  if ((e = launch_amax(x, M * K, ws, s, sms, status, timeout())) != cudaSuccess) return e;
+  return launch_quant_nvfp4(x, M, K, reinterpret_cast<const float*>(ws), true, out, s, sms, status,
+                            timeout());
+}
+
 }  // namespace qlin
 
 using namespace qlin;
@@ -147,10 +158,8 @@ qlin_status qlin_quantize_act_nvfp4(const void* x_bf16, int64_t M, int64_t K,
   QLIN_TRY(device_state(&status, &sms));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (static_scale == nullptr) {
-    unsigned* amax = static_cast<unsigned*>(workspace);
-    QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms, status, timeout()));
-    QLIN_CUDA(launch_quant_nvfp4(x_bf16, M, K, reinterpret_cast<const float*>(amax), true, *out,
-                                 s, sms, status, timeout()));
+    QLIN_CUDA(quant_nvfp4_dynamic(x_bf16, M, K, *out, static_cast<unsigned*>(workspace), s, sms,
+                                  status));
   } else {
     QLIN_CUDA(launch_quant_nvfp4(x_bf16, M, K, static_scale, false, *out, s, sms, status, timeout()));
   }
@@ -174,10 +183,9 @@ qlin_status qlin_quantize_act_nvfp4_noalloc(const void* x_bf16, int64_t M, int64
   unsigned char* scratch = nullptr;
   QLIN_TRY(noalloc_scratch(&scratch));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  unsigned* amax = reinterpret_cast<unsigned*>(scratch);  // cleared by launch_amax
-  QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms, status, timeout()));
-  QLIN_CUDA(launch_quant_nvfp4(x_bf16, M, K, reinterpret_cast<const float*>(amax), true, *out, s,
-                               sms, status, timeout()));
+  // the scratch words are cleared by the launch that uses them
+  QLIN_CUDA(quant_nvfp4_dynamic(x_bf16, M, K, *out, reinterpret_cast<unsigned*>(scratch), s, sms,
+                                status));
   return QLIN_OK;
 }
 
@@ -195,10 +203,14 @@ qlin_status qlin_quantize_act_fp8(const void* x_bf16, int64_t M, int64_t K,
   QLIN_TRY(device_state(&status, &sms));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (static_scale == nullptr) {
-    unsigned* amax = static_cast<unsigned*>(workspace);
-    QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms, status, timeout()));
-    QLIN_CUDA(launch_quant_fp8(x_bf16, M, K, reinterpret_cast<const float*>(amax), true, *out, s,
-                               sms, status, timeout()));
+    unsigned* ws = static_cast<unsigned*>(workspace);
+    cudaError_t e = launch_quant_fp8_onepass(x_bf16, M, K, *out, ws, s, sms, status, timeout());
+    if (e == cudaErrorNotSupported) {   // x does not fit on chip: amax pass, then quantize
+      QLIN_CUDA(launch_amax(x_bf16, M * K, ws, s, sms, status, timeout()));
+      e = launch_quant_fp8(x_bf16, M, K, reinterpret_cast<const float*>(ws), true, *out, s, sms,
+                           status, timeout());
+    }
+    QLIN_CUDA(e);
   } else {
     QLIN_CUDA(launch_quant_fp8(x_bf16, M, K, static_scale, false, *out, s, sms, status, timeout()));
   }

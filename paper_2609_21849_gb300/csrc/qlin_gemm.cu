@@ -565,7 +565,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // No CTA of the cluster may exit while a peer can still multicast into it
-  // or arrive on its barriers.
+  // or arrive on its barriers.  Each warp reconverges first: the cluster
+  // barrier is a warp-aligned instruction, and most roles run on one lane.
+  __syncwarp();
   tc_fence_before();
   if (kPair)
     cluster_sync();

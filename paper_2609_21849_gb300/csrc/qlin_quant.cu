@@ -2,6 +2,9 @@
 // post-training quantization; activations are quantized at run time, weights
 // once).  All kernels here are HBM-bandwidth bound streaming kernels:
 //
+//   onepass_kernel<Op>    dynamic scale in one read of x: the grid holds x in
+//                         shared memory, reduces amax across the grid, then
+//                         quantizes from shared memory (when x fits on chip)
 //   amax_kernel           max |x| over a tensor (the dynamic tensor scale)
 //   quant_kernel<NVFP4>   bf16 -> packed e2m1 codes + E4M3 block scales in the
 //                         tensor-core scale layout + FP32 tensor scale
@@ -54,6 +57,7 @@ __device__ __forceinline__ uint4 lds128(const uint4* p) {
 struct AmaxOp {
   static constexpr int kUnit = 1;   // chunks per thread and call
   uint32_t m = 0;
+  __device__ __forceinline__ void bind(float*) {}
   __device__ __forceinline__ void init() {}
   __device__ __forceinline__ void unit(const uint4 (&v)[1], uint64_t, bool valid) {
     if (valid) m = max(m, chunk_abs_max_bits(v[0]));
@@ -72,14 +76,17 @@ struct Nvfp4Op {
   uint32_t* codes;
   uint8_t* scales;
   float* r_table;   // shared memory, 128 entries
+  __device__ __forceinline__ void bind(float* table) { r_table = table; }
   __device__ __forceinline__ void init() {
     if (threadIdx.x < 128) {
       const uint32_t c = threadIdx.x;
       r_table[c] = (c == 0u) ? 0.0f : __fdiv_rn(s_enc, e4m3_value(c));
     }
   }
-  __device__ __forceinline__ void unit(const uint4 (&v)[2], uint64_t c, bool valid) {
-    const int lane = threadIdx.x & 31;
+  // The codes of one 16-element block and its scale code; lanes 4g..4g+3
+  // hold one 64-element group, whose four scales are gathered into lane 4g.
+  __device__ __forceinline__ void quantize_block(const uint4 (&v)[2], uint32_t& code0,
+                                                 uint32_t& code1, uint32_t& word) const {
     const uint32_t mb = max(chunk_abs_max_bits(v[0]), chunk_abs_max_bits(v[1]));
     const float t = __fmul_rn(__uint_as_float(mb << 16), s_enc);
     const uint32_t sb = e4m3_code(__fdiv_rn(t, 6.0f));
@@ -88,23 +95,79 @@ struct Nvfp4Op {
     unpack8(v[0], f);
 #pragma unroll
     for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], r_b);
-    const uint32_t code0 = e2m1x8(f);
+    code0 = e2m1x8(f);
     unpack8(v[1], f);
 #pragma unroll
     for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], r_b);
-    const uint32_t code1 = e2m1x8(f);
-    // gather the group's four scales into its first lane
+    code1 = e2m1x8(f);
     const uint32_t s1 = __shfl_down_sync(0xFFFFFFFFu, sb, 1);
     const uint32_t s2 = __shfl_down_sync(0xFFFFFFFFu, sb, 2);
     const uint32_t s3 = __shfl_down_sync(0xFFFFFFFFu, sb, 3);
+    word = sb | (s1 << 8) | (s2 << 16) | (s3 << 24);
+  }
+  __device__ __forceinline__ void unit(const uint4 (&v)[2], uint64_t c, bool valid) {
+    uint32_t code0, code1, word;
+    quantize_block(v, code0, code1, word);
     if (valid) {
       reinterpret_cast<uint2*>(codes)[c >> 1] = make_uint2(code0, code1);
-      if ((lane & 3) == 0) {
+      if ((threadIdx.x & 3) == 0) {
         const Idx ci = (Idx)c;
         const Idx row = ci / chunks_per_row;
         const Idx col = (ci - row * chunks_per_row) << 3;
         *reinterpret_cast<uint32_t*>(scales + scale_offset((int64_t)row, (int64_t)(col >> 4), K)) =
-            sb | (s1 << 8) | (s2 << 16) | (s3 << 24);
+            word;
+      }
+    }
+  }
+  // A slice of n chunks held in shared memory, global chunks [c0, c0 + n)
+  // (c0 and n multiples of 8): each thread takes units of two chunks at a
+  // stride of the block, two units per step for instruction-level
+  // parallelism, and tracks its row and column without dividing.
+  template <int kThreadsPerBlock>
+  __device__ __forceinline__ void run_slice(const uint4* buf, uint32_t n, uint64_t c0) const {
+    constexpr uint32_t kStride = 2u * kThreadsPerBlock;          // chunks per step and unit
+    const uint32_t cpr = (uint32_t)chunks_per_row;
+    const uint32_t dq = (2u * kStride) / cpr, dr = (2u * kStride) % cpr;
+    const uint32_t kq = kStride / cpr, kr = kStride % cpr;
+    const uint64_t cg = c0 + 2u * threadIdx.x;
+    uint32_t row = (uint32_t)(cg / cpr), col = (uint32_t)(cg % cpr);   // col in chunks
+    const uint32_t kgroups = (uint32_t)(K >> 6);
+    // the loop bound is block-uniform: every lane reaches the shuffles
+    for (uint32_t base = 0; base < n; base += 2u * kStride) {
+      const uint32_t cl = base + 2u * threadIdx.x;
+      uint4 va[2], vb[2];
+      const bool ok_a = cl < n, ok_b = cl + kStride < n;   // units never straddle n
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        va[k] = ok_a ? lds128(buf + cl + k) : make_uint4(0u, 0u, 0u, 0u);
+        vb[k] = ok_b ? lds128(buf + cl + kStride + k) : make_uint4(0u, 0u, 0u, 0u);
+      }
+      uint32_t a0, a1, aw, b0, b1, bw;
+      quantize_block(va, a0, a1, aw);
+      quantize_block(vb, b0, b1, bw);
+      uint32_t row_b = row + kq, col_b = col + kr;
+      if (col_b >= cpr) {
+        col_b -= cpr;
+        ++row_b;
+      }
+      const bool lead = (threadIdx.x & 3) == 0;
+      if (ok_a) {
+        reinterpret_cast<uint2*>(codes)[(c0 + cl) >> 1] = make_uint2(a0, a1);
+        if (lead)
+          *reinterpret_cast<uint32_t*>(scales + ((row >> 7) * kgroups + (col >> 3)) * 512u +
+                                       (row & 31u) * 16u + ((row >> 5) & 3u) * 4u) = aw;
+      }
+      if (ok_b) {
+        reinterpret_cast<uint2*>(codes)[(c0 + cl + kStride) >> 1] = make_uint2(b0, b1);
+        if (lead)
+          *reinterpret_cast<uint32_t*>(scales + ((row_b >> 7) * kgroups + (col_b >> 3)) * 512u +
+                                       (row_b & 31u) * 16u + ((row_b >> 5) & 3u) * 4u) = bw;
+      }
+      row += dq;
+      col += dr;
+      if (col >= cpr) {
+        col -= cpr;
+        ++row;
       }
     }
   }
@@ -114,6 +177,7 @@ struct Fp8Op {
   static constexpr int kUnit = 1;
   float s_enc;
   uint2* codes;
+  __device__ __forceinline__ void bind(float*) {}
   __device__ __forceinline__ void init() {}
   __device__ __forceinline__ void unit(const uint4 (&v)[1], uint64_t c, bool valid) {
     if (!valid) return;
@@ -122,6 +186,17 @@ struct Fp8Op {
 #pragma unroll
     for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], s_enc);
     codes[c] = make_uint2(e4m3x4(f[0], f[1], f[2], f[3]), e4m3x4(f[4], f[5], f[6], f[7]));
+  }
+  template <int kThreadsPerBlock>
+  __device__ __forceinline__ void run_slice(const uint4* buf, uint32_t n, uint64_t c0) const {
+    for (uint32_t cl = threadIdx.x; cl < n; cl += kThreadsPerBlock) {
+      float f[8];
+      unpack8(lds128(buf + cl), f);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], s_enc);
+      codes[c0 + cl] =
+          make_uint2(e4m3x4(f[0], f[1], f[2], f[3]), e4m3x4(f[4], f[5], f[6], f[7]));
+    }
   }
 };
 
@@ -307,6 +382,85 @@ __global__ void __launch_bounds__(kThreads) quant_fp8_rows_kernel(const uint4* _
   }
 }
 
+// ------------------------------------------------ one-pass dynamic scale ---
+// The tensor scale depends on max |x| over the whole tensor (the amax pass),
+// and the codes depend on the tensor scale, so a streaming quantizer reads x
+// twice.  When x fits in the aggregate shared memory of the grid (one CTA per
+// SM, launched cooperatively so every CTA is resident), each CTA loads its
+// slice once, the grid combines the slice maxima through two words of
+// global memory, and each CTA quantizes its slice from shared memory.
+constexpr int kOnePassThreads = 1024;
+constexpr int kOnePassSmem = 225 * 1024;
+constexpr int kOnePassSliceMax = 14 * 1024;       // chunks: 224 KB of data at most
+
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const unsigned* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// sync[0]: amax bits (fp32), sync[1]: arrival count; both zero at launch.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+
+// sync[0]: amax bits (fp32), sync[1]: arrival count; both zero at launch.
+template <typename Op>
+__global__ void __launch_bounds__(kOnePassThreads, 1)
+    onepass_kernel(const uint4* __restrict__ x, uint64_t n_chunks, uint32_t slice, Op op,
+                   float qmax, float* sdec_out, unsigned* sync, unsigned* err,
+                   uint64_t timeout_ns) {
+  extern __shared__ __align__(128) uint8_t qsm[];
+  uint4* buf = reinterpret_cast<uint4*>(qsm);
+  __shared__ uint32_t warp_max[kOnePassThreads / 32];
+  __shared__ float op_table[128];
+  __shared__ float s_amax;
+  __shared__ int abort_flag;
+  const int tid = threadIdx.x;
+  const uint64_t c_begin = (uint64_t)blockIdx.x * slice;
+  const uint32_t n = c_begin >= n_chunks ? 0u
+                     : (uint32_t)(n_chunks - c_begin < slice ? n_chunks - c_begin : slice);
+  // every thread copies its chunks (a dozen 16-byte asynchronous copies in
+  // flight per thread), then takes their amax
+  const uint4* xs = x + c_begin;
+  for (uint32_t i = tid; i < n; i += kOnePassThreads) cp_async16(smem_u32(buf + i), xs + i);
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
+  uint32_t m = 0;
+  for (uint32_t i = tid; i < n; i += kOnePassThreads) m = max(m, chunk_abs_max_bits(lds128(buf + i)));
+  m = __reduce_max_sync(0xFFFFFFFFu, m);
+  if ((tid & 31) == 0) warp_max[tid >> 5] = m;
+  if (tid == 0) abort_flag = 0;
+  __syncthreads();
+  if (tid == 0) {
+    uint32_t b = 0;
+#pragma unroll
+    for (int w = 0; w < kOnePassThreads / 32; ++w) b = max(b, warp_max[w]);
+    // publish, arrive, and wait (bounded) for every CTA of the grid
+    if (b) atomicMax(&sync[0], b << 16);
+    // the arrival releases the maximum above to every CTA that sees it
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(&sync[1]) : "memory");
+    const uint64_t t0 = global_timer_ns();
+    while (ld_acquire_gpu(&sync[1]) < gridDim.x) {
+      if (global_timer_ns() - t0 > timeout_ns) {
+        atomicExch(err, kErrTimeout);
+        abort_flag = 1;
+        break;
+      }
+    }
+    s_amax = __uint_as_float(ld_acquire_gpu(&sync[0]));
+  }
+  __syncthreads();
+  if (abort_flag) return;
+  const float amax = s_amax;
+  const float s_dec = (amax == 0.0f) ? 1.0f : __fdiv_rn(amax, qmax);
+  if (blockIdx.x == 0 && tid == 0) *sdec_out = s_dec;
+  op.s_enc = encode_scale(s_dec);
+  op.bind(op_table);
+  op.init();
+  __syncthreads();
+  op.template run_slice<kOnePassThreads>(buf, n, c_begin);
+}
+
 // Opt each kernel into kSmem bytes of dynamic shared memory, once.
 template <auto kKern>
 cudaError_t set_smem() {
@@ -331,6 +485,73 @@ cudaError_t launch_amax(const void* x, int64_t n_elems, unsigned* amax_bits, cud
   amax_kernel<<<stream_grid(n_chunks, num_sms), kThreads, kSmem, s>>>(
       static_cast<const uint4*>(x), n_chunks, amax_bits, err, timeout_ns);
   return cudaGetLastError();
+}
+
+// One-pass dynamic quantization when x fits on chip: returns
+// cudaErrorNotSupported (nothing launched) when it does not, or when the
+// device cannot hold the grid resident.
+template <typename Op>
+static cudaError_t launch_onepass(const void* x, uint64_t n_chunks, const Op& op, float qmax,
+                                  float* sdec_out, unsigned* sync, cudaStream_t s, int num_sms,
+                                  unsigned* err, uint64_t timeout_ns) {
+  // slices of whole 64-element groups (8 chunks), one per SM
+  uint64_t slice = (n_chunks + num_sms - 1) / num_sms;
+  slice = (slice + 7) / 8 * 8;
+  if (slice > (uint64_t)kOnePassSliceMax || slice == 0) return cudaErrorNotSupported;
+  const int grid = (int)((n_chunks + slice - 1) / slice);
+  auto kern = onepass_kernel<Op>;
+  static const cudaError_t attr =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kOnePassSmem);
+  if (attr != cudaSuccess) return attr;
+  static int resident = -1;   // CTAs of this kernel one SM can hold
+  if (resident < 0) {
+    int r = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, kern, kOnePassThreads, kOnePassSmem) !=
+        cudaSuccess)
+      r = 0;
+    resident = r;
+  }
+  if (resident < 1 || grid > num_sms * resident) return cudaErrorNotSupported;
+  cudaError_t e = cudaMemsetAsync(sync, 0, 2 * sizeof(unsigned), s);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg{};
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeCooperative;   // all CTAs resident: the grid waits on itself
+  at[0].val.cooperative = 1;
+  cfg.gridDim = dim3((unsigned)grid, 1, 1);
+  cfg.blockDim = dim3(kOnePassThreads, 1, 1);
+  cfg.dynamicSmemBytes = kOnePassSmem;
+  cfg.stream = s;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<const uint4*>(x), n_chunks, (uint32_t)slice,
+                            op, qmax, sdec_out, sync, err, timeout_ns);
+}
+
+cudaError_t launch_quant_nvfp4_onepass(const void* x, int64_t M, int64_t K,
+                                       const qlin_nvfp4_t& out, unsigned* sync, cudaStream_t s,
+                                       int num_sms, unsigned* err, uint64_t timeout_ns) {
+  const uint64_t n_chunks = (uint64_t)M * (uint64_t)K / 8;
+  if (n_chunks >= (1ull << 32)) return cudaErrorNotSupported;
+  Nvfp4Op<uint32_t> op;
+  op.s_enc = 0.0f;   // set in the kernel once amax is known
+  op.chunks_per_row = (uint32_t)(K >> 3);
+  op.K = K;
+  op.codes = reinterpret_cast<uint32_t*>(out.codes);
+  op.scales = out.scales;
+  op.r_table = nullptr;   // set in the kernel (shared memory)
+  return launch_onepass(x, n_chunks, op, 2688.0f, out.tensor_scale, sync, s, num_sms, err,
+                        timeout_ns);
+}
+
+cudaError_t launch_quant_fp8_onepass(const void* x, int64_t M, int64_t K, const qlin_fp8_t& out,
+                                     unsigned* sync, cudaStream_t s, int num_sms, unsigned* err,
+                                     uint64_t timeout_ns) {
+  const uint64_t n_chunks = (uint64_t)M * (uint64_t)K / 8;
+  Fp8Op op;
+  op.s_enc = 0.0f;
+  op.codes = reinterpret_cast<uint2*>(out.codes);
+  return launch_onepass(x, n_chunks, op, 448.0f, out.scale, sync, s, num_sms, err, timeout_ns);
 }
 
 template <bool kDynamic>

@@ -126,3 +126,37 @@ def test_fp8_weight_per_channel(N, K):
     q = qlin.qlin_quantize_weight(to_dev(w), qlin.QLIN_FMT_FP8)
     assert np.array_equal(f32(q.scale).view(np.uint32), rs.view(np.uint32))
     assert np.array_equal(u8(q.codes), rc)
+
+
+@pytest.mark.parametrize("fmt", ["nvfp4", "fp8"])
+def test_dynamic_scale_x_larger_than_on_chip(fmt):
+    # 9216 x 4096 bf16 (75.5 MB) exceeds what the grid can hold on chip, so
+    # the dynamic scale takes the amax pass + quantizer route; the 4608 x 3072
+    # cases above take the one-read route.  Both must equal the oracle.
+    M, K = 9216, 4096
+    x = synthetic.act_entry_outliers(77, M, K)
+    if fmt == "nvfp4":
+        q = qlin.qlin_quantize_act_nvfp4(to_dev(x))
+        assert qlin.qlin_sync_status() == 0
+        assert_nvfp4_equal(q, oracle.quant_nvfp4(x), "9216x4096 dynamic")
+    else:
+        rc, rs = oracle.quant_fp8(x)
+        q = qlin.qlin_quantize_act_fp8(to_dev(x))
+        assert qlin.qlin_sync_status() == 0
+        assert f32(q.scale)[0].view(np.uint32) == np.float32(rs).view(np.uint32)
+        assert np.array_equal(u8(q.codes), rc)
+
+
+def test_dynamic_scale_one_read_repeated():
+    # the one-read route keeps its grid-wide amax in two scratch words that
+    # each launch clears: back-to-back calls on tensors of decreasing amax
+    # must not see a stale maximum
+    M, K = 4608, 3072
+    ws = qlin.alloc_workspace()
+    for seed, gain in ((5, 8.0), (6, 1.0), (7, 0.125)):
+        x = (synthetic.act_normal(seed, M, K).view(np.uint16))
+        xf = (x.astype(np.uint32) << 16).view(np.float32) * np.float32(gain)
+        xb = synthetic.bf16_bits(xf)
+        q = qlin.qlin_quantize_act_nvfp4(to_dev(xb), None, qlin.alloc_nvfp4(M, K), ws)
+        assert qlin.qlin_sync_status() == 0
+        assert_nvfp4_equal(q, oracle.quant_nvfp4(xb), f"gain {gain}")
