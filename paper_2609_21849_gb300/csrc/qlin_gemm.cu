@@ -356,10 +356,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 2 || warp == 3) {
     // --------------------------------------------- NVFP4 scale copies ---
-    // Block scales move shared -> TMEM from two threads of their own (a
-    // tcgen05.cp occupies its issuing thread ~50 cycles), beside the MMA
-    // stream: warp 2 the A atoms and W atom row 0, warp 3 W atom row 1.  In a
-    // pair, CTA 0's copies fill both SMs' TMEM from their own shared memory.
+    // Block scales move shared -> TMEM from two threads of their own, beside
+    // the MMA stream: a tcgen05.cp occupies its issuing thread ~90-120 cycles
+    // while the MMAs run, and a stage needs 12 (pair tiles), so warp 2 copies
+    // the atoms of the stage's first two MMA steps and warp 3 those of the
+    // last two.  In a pair, CTA 0's copies fill both SMs' TMEM from their own
+    // shared memory.
     if (kFp4 && lane == 0 && leader) {
       const int sw = warp - 2;
       int stage = 0;
@@ -375,24 +377,26 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t sSFA = smem_u32(smem + stage * C::kStageBytes) + C::kABytes + C::kBBytes;
           const uint32_t sSFB = sSFA + C::kSfaBytes;
           const int nsteps = min(kStepsPerStage, k_steps - kb * kStepsPerStage);
-          for (int j = 0; j < nsteps; ++j) {
+          // each warp copies all atoms (A, then each W atom row) of half the
+          // stage's MMA steps
+          constexpr int kHalf = kStepsPerStage / 2;
+          const int j_end = min(nsteps, (sw + 1) * kHalf);
+          for (int j = sw * kHalf; j < j_end; ++j) {
             const uint32_t sfa_t = tmem_base + (uint32_t)(C::kSfColBase +
                                                           (stage * kStepsPerStage + j) *
                                                               C::kSfColsPerStep);
-            if (sw == 0) {
-              if (kPair) {
-                tc_cp_scales_pair(sfa_t, sdesc_scales(sSFA + j * 512));
-                tc_cp_scales_pair(sfa_t + 4, sdesc_scales(sSFB + j * 512));
-              } else {
-                tc_cp_scales(sfa_t, sdesc_scales(sSFA + j * 512));
-                tc_cp_scales(sfa_t + 4, sdesc_scales(sSFB + j * 512));
-              }
-            } else if (C::kSfbAtoms > 1) {
+            if (kPair)
+              tc_cp_scales_pair(sfa_t, sdesc_scales(sSFA + j * 512));
+            else
+              tc_cp_scales(sfa_t, sdesc_scales(sSFA + j * 512));
+#pragma unroll
+            for (int r = 0; r < C::kSfbAtoms; ++r) {
               if (kPair)
-                tc_cp_scales_pair(sfa_t + 8,
-                                  sdesc_scales(sSFB + kStepsPerStage * 512 + j * 512));
+                tc_cp_scales_pair(sfa_t + 4 + 4 * r,
+                                  sdesc_scales(sSFB + r * kStepsPerStage * 512 + j * 512));
               else
-                tc_cp_scales(sfa_t + 8, sdesc_scales(sSFB + kStepsPerStage * 512 + j * 512));
+                tc_cp_scales(sfa_t + 4 + 4 * r,
+                             sdesc_scales(sSFB + r * kStepsPerStage * 512 + j * 512));
             }
           }
           if (kPair)
