@@ -10,7 +10,7 @@
 //          drives both SMs' tensor cores; each CTA holds its own 128 rows of A
 //          and its own half of the W tile in shared memory.
 //   single 128 x 128 tiles on one CTA, for small M (the translator's linears).
-// Roles (12 warps, one persistent CTA per SM):
+// Roles (one persistent CTA per SM; 12 warps, 14 for NVFP4 pair tiles):
 //   warp 0      TMA producer: per pipeline stage one 4-D tensor copy per lane
 //               (A tile, W tile, A scale atoms, W scale atoms), issued by four
 //               lanes as a single instruction.  In a pair, CTA 1's copies
@@ -18,9 +18,9 @@
 //   warp 1      TMEM allocation; MMA issue (per 32 bytes of K one tcgen05.mma:
 //               NVFP4 kind::mxf4nvf4 scale_vec::4X with K = 64, FP8
 //               kind::f8f6f4 with K = 32) into an fp32 TMEM accumulator.
-//   warps 2-3   NVFP4: block scales shared -> TMEM (tcgen05.cp), beside the
-//               MMA stream.
-//   warps 4-11  epilogue: tcgen05.ld of the accumulator, alpha, bf16, TMA
+//   warps 2..   NVFP4: block scales shared -> TMEM (tcgen05.cp), beside the
+//               MMA stream (two warps, four for pair tiles).
+//   last 8      epilogue: tcgen05.ld of the accumulator, alpha, bf16, TMA
 //               stores through swizzled staging, optional NVFP4 re-quantization
 //               of the bf16 values (one row per thread).
 // Every wait is bounded (see WaitCtl).
@@ -37,8 +37,12 @@ constexpr int kBM = 128;
 constexpr int kRowBytes = 128;      // bytes of K per stage and row: one swizzle row
 constexpr int kStepsPerStage = 4;   // one MMA per 32 bytes of K
 constexpr int kEpiWarps = 8;
-constexpr int kEpiWarp0 = 4;   // warps 0-3: producer, MMA, two scale-copy warps
-constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
+#ifndef QLIN_PAIR_CP_WARPS
+#define QLIN_PAIR_CP_WARPS 2
+#endif
+#ifndef QLIN_SPLIT_SCALE_ISSUE
+#define QLIN_SPLIT_SCALE_ISSUE 1
+#endif
 constexpr int kSmemBudget = 232448 - 2048;  // opt-in shared memory minus barriers/alignment
 #ifndef QLIN_TMA_SPLIT
 #define QLIN_TMA_SPLIT 1
@@ -55,6 +59,16 @@ constexpr int pow2_at_least(int x) {
 // holds its own 128 rows of A and its own half of the W tile.
 template <bool kFp4, int kBN, bool kPair = false>
 struct Cfg {
+  // warps: 0 producer, 1 MMA, then the scale-copy warps, then the epilogue
+  // (an epilogue warp w reads TMEM lanes 32 (w % 4) and up, so any eight
+  // consecutive warps cover the accumulator).  NVFP4 pair tiles need 12
+  // scale copies per stage, more than two warps issue in an MMA stage.
+  static constexpr int kCpWarps = (kFp4 && kPair) ? QLIN_PAIR_CP_WARPS : 2;
+  // NVFP4 pair tiles: a warp of its own issues the scale boxes, so the
+  // operand boxes' instruction has two lanes instead of four
+  static constexpr int kScaleWarp = (kFp4 && kPair && QLIN_SPLIT_SCALE_ISSUE) ? 2 + kCpWarps : -1;
+  static constexpr int kEpiWarp0 = 2 + kCpWarps + (kScaleWarp >= 0 ? 1 : 0);
+  static constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
   static constexpr int kSfbAtoms = kFp4 ? (kBN + 127) / 128 : 0;
   static constexpr int kABytes = kBM * kRowBytes;
   static constexpr int kBBytes = (kPair ? kBN / 2 : kBN) * kRowBytes;
@@ -117,7 +131,7 @@ __device__ __forceinline__ void st_global_v4(void* p, uint32_t a, uint32_t b, ui
 }
 
 template <bool kFp4, int kBN, bool kPair, bool kRequant>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_a,
                 const __grid_constant__ CUtensorMap tmap_b,
                 const __grid_constant__ CUtensorMap tmap_sfa,
@@ -137,8 +151,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* tmem_full = sf_full + C::kStages;
   uint64_t* tmem_empty = tmem_full + 2;
   uint64_t* mma_done = tmem_empty + 2;
-  uint64_t* sf_done = mma_done + 1;   // two barriers, one per scale-copy warp
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sf_done + 2);
+  uint64_t* sf_done = mma_done + 1;   // one barrier per scale-copy warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sf_done + C::kCpWarps);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -150,7 +164,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
-      mbar_init(&sf_ready[s], 2);   // one commit per scale-copy warp
+      mbar_init(&sf_ready[s], C::kCpWarps);   // one commit per scale-copy warp
       mbar_init(&sf_full[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -158,8 +172,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&tmem_empty[a], kCM * kEpiWarps);   // every epilogue warp of the cluster
     }
     mbar_init(mma_done, 1);
-    mbar_init(&sf_done[0], 1);
-    mbar_init(&sf_done[1], 1);
+    for (int w = 0; w < C::kCpWarps; ++w) mbar_init(&sf_done[w], 1);
     *abort_flag = 0;
     mbar_fence_init();
   }
@@ -190,7 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int num_kb = (int)((k_bytes + kRowBytes - 1) / kRowBytes);
   const int k_steps = (int)(k_bytes / 32);
 
-  if (warp == 0) {
+  if (warp == 0 || warp == C::kScaleWarp) {
     // ------------------------------------------------------ TMA producer ---
     // One 4-D tensor copy per lane (0: A tile, 1: W tile, 2: A scale atoms,
     // 3: W scale atoms), all four issued as ONE instruction: a TMA copy holds
@@ -201,15 +214,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Each operand tile is split into kSplit row boxes, one lane each, so
     // more copies run at once (lanes [0, kSplit): A parts, [kSplit, 2 kSplit):
     // W parts, then A scales, W scales).
+    // With a scale-issue warp, warp 0 takes the operand lanes and that warp
+    // the two scale lanes; pl numbers the producer lanes across both.
     constexpr int kOpLanes = 2 * kSplit;
-    const int nlanes = kFp4 ? kOpLanes + 2 : kOpLanes;
+    const int pl = warp == 0 ? lane : kOpLanes + lane;
+    const int nlanes = warp != 0 ? 2 : (kFp4 && C::kScaleWarp < 0) ? kOpLanes + 2 : kOpLanes;
     if (lane < nlanes) {
-      const bool is_scale = lane >= kOpLanes;
-      const int part = lane % kSplit;
-      const CUtensorMap* map = lane < kSplit      ? &tmap_a
-                               : lane < kOpLanes  ? &tmap_b
-                               : lane == kOpLanes ? &tmap_sfa
-                                                  : &tmap_sfb;
+      const bool is_scale = pl >= kOpLanes;
+      const int part = pl % kSplit;
+      const CUtensorMap* map = pl < kSplit      ? &tmap_a
+                               : pl < kOpLanes  ? &tmap_b
+                               : pl == kOpLanes ? &tmap_sfa
+                                                : &tmap_sfb;
       uint64_t* bars = is_scale ? sf_full : full;
       // barrier each copy completes on: this CTA's, or in a pair CTA 0's
       const uint32_t bar0 = kPair ? mapa_shared(bars, 0) : smem_u32(bars);
@@ -227,22 +243,22 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           uint8_t* sA = smem + stage * C::kStageBytes;
           uint8_t* sB = sA + C::kABytes;
-          if (leader && lane == 0)
+          if (leader && pl == 0)
             mbar_arrive_expect_tx(&full[stage], kCM * (C::kABytes + C::kBBytes));
-          if (kFp4 && leader && lane == kOpLanes)
+          if (kFp4 && leader && pl == kOpLanes)
             mbar_arrive_expect_tx(&sf_full[stage], kCM * (C::kSfaBytes + C::kSfbBytes));
           __syncwarp((1u << nlanes) - 1u);
           uint8_t* dst;
           int32_t c0, c1, c2, c3;
           constexpr int kARows = kBM / kSplit, kBRowsPart = kBN / kCM / kSplit;
-          if (lane < kSplit) {              // A: part of this CTA's M tile
+          if (pl < kSplit) {                // A: part of this CTA's M tile
             dst = sA + part * kARows * kRowBytes;
             c0 = kb * kRowBytes; c1 = mb * kBM + part * kARows; c2 = 0; c3 = 0;
-          } else if (lane < kOpLanes) {     // W: part of this CTA's rows of the N tile
+          } else if (pl < kOpLanes) {       // W: part of this CTA's rows of the N tile
             dst = sB + part * kBRowsPart * kRowBytes;
             c0 = kb * kRowBytes; c1 = nb * kBN + rank * (kBN / kCM) + part * kBRowsPart;
             c2 = 0; c3 = 0;
-          } else if (lane == kOpLanes) {    // A scale atoms of this stage
+          } else if (pl == kOpLanes) {      // A scale atoms of this stage
             dst = sB + C::kBBytes; c0 = kb * kStepsPerStage * 64; c1 = mb; c2 = 0; c3 = 0;
           } else {                          // W scale atoms (all atom rows of the N tile)
             dst = sB + C::kBBytes + C::kSfaBytes; c0 = kb * kStepsPerStage * 64;
@@ -263,7 +279,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // Let the last copies into this CTA land before it exits (the barriers
       // that count them live in CTA 0; its producer drains them).
-      if (leader && (lane == 0 || (kFp4 && lane == kOpLanes))) {
+      if (leader && (pl == 0 || (kFp4 && pl == kOpLanes))) {
         const int n_drain = min(issued, C::kStages);
         for (int i = 0; i < n_drain; ++i) {
           if (--stage < 0) {
@@ -354,14 +370,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_commit(mma_done);
       mbar_drain(mma_done, 0, p.timeout_ns, p.err);
     }
-  } else if (warp == 2 || warp == 3) {
+  } else if (warp < C::kEpiWarp0) {
     // --------------------------------------------- NVFP4 scale copies ---
-    // Block scales move shared -> TMEM from two threads of their own, beside
-    // the MMA stream: a tcgen05.cp occupies its issuing thread ~90-120 cycles
-    // while the MMAs run, and a stage needs 12 (pair tiles), so warp 2 copies
-    // the atoms of the stage's first two MMA steps and warp 3 those of the
-    // last two.  In a pair, CTA 0's copies fill both SMs' TMEM from their own
-    // shared memory.
+    // Block scales move shared -> TMEM from threads of their own (one lane of
+    // each scale-copy warp), beside the MMA stream: a tcgen05.cp occupies its
+    // issuing thread ~80-120 cycles while the MMAs run, and a stage needs 12
+    // (pair tiles), so each warp copies the atoms of an equal share of the
+    // stage's MMA steps.  In a pair, CTA 0's copies fill both SMs' TMEM from
+    // their own shared memory.
     if (kFp4 && lane == 0 && leader) {
       const int sw = warp - 2;
       int stage = 0;
@@ -377,11 +393,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t sSFA = smem_u32(smem + stage * C::kStageBytes) + C::kABytes + C::kBBytes;
           const uint32_t sSFB = sSFA + C::kSfaBytes;
           const int nsteps = min(kStepsPerStage, k_steps - kb * kStepsPerStage);
-          // each warp copies all atoms (A, then each W atom row) of half the
-          // stage's MMA steps
-          constexpr int kHalf = kStepsPerStage / 2;
-          const int j_end = min(nsteps, (sw + 1) * kHalf);
-          for (int j = sw * kHalf; j < j_end; ++j) {
+          // each warp copies all atoms (A, then each W atom row) of its share
+          // of the stage's MMA steps
+          constexpr int kShare = kStepsPerStage / C::kCpWarps;
+          const int j_end = min(nsteps, (sw + 1) * kShare);
+          for (int j = sw * kShare; j < j_end; ++j) {
             const uint32_t sfa_t = tmem_base + (uint32_t)(C::kSfColBase +
                                                           (stage * kStepsPerStage + j) *
                                                               C::kSfColsPerStep);
@@ -420,7 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // --------------------------------------------------------- epilogue ---
     constexpr int kCols = kBN / 2;  // columns per thread
     constexpr int kChunks = kCols / 32;
-    const int e = warp - kEpiWarp0;
+    const int e = warp - C::kEpiWarp0;
     const int quarter = warp & 3;   // the TMEM lane quarter this warp may access
     const int half = e >> 2;
     uint8_t* const out_buf = out_stage + e * 4096;   // this warp's two staging boxes
@@ -430,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (kRequant) {
       const float s_next = *p.next_scale;
       s_enc_next = encode_scale(s_next);
-      if (blockIdx.x == 0 && threadIdx.x == kEpiWarp0 * 32 && p.rq_tensor_scale != p.next_scale)
+      if (blockIdx.x == 0 && threadIdx.x == C::kEpiWarp0 * 32 && p.rq_tensor_scale != p.next_scale)
         *p.rq_tensor_scale = s_next;
     }
     int acc = 0;
@@ -447,9 +463,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * kBN + half * kCols);
       // Accumulator columns in batches of tcgen05.ld per wait; TMEM goes back
       // to the MMA issuer right after the last batch has landed in registers.
-      // With a single accumulator (NVFP4 pair tiles) the next tile's MMAs
-      // wait for that, so there all columns form one batch.
-      constexpr int kBatch = C::kNumAcc == 1 ? kChunks : 2;
+      // With a single accumulator the next tile's MMAs wait for that, so all
+      // columns form one batch where the register budget (168 a thread at
+      // 12 warps, 128 above) allows.
+      constexpr int kBatch = (C::kNumAcc == 1 && C::kThreads <= 384) ? kChunks : 2;
 #pragma unroll
       for (int cb = 0; cb < kChunks; cb += kBatch) {
         uint32_t r[kBatch][32];
@@ -705,7 +722,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   attr[0].val.clusterDim.x = kCM;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.blockDim = dim3(C::kThreads, 1, 1);
   cfg.dynamicSmemBytes = C::kSmemBytes;
   cfg.stream = s;
   cfg.attrs = attr;
