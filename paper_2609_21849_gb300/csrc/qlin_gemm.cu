@@ -592,7 +592,10 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
         }
       }
     }
-    if (lane == 0) bulk_wait_group_all();   // output stores complete before exit
+    // The staging buffers must have been read out before the CTA exits; the
+    // stores' global writes complete with the grid (as for any store), so
+    // the CTA does not wait for them.
+    if (lane == 0) bulk_wait_group_read<0>();
   }
 
   // No CTA of the cluster may exit while a peer can still multicast into it
