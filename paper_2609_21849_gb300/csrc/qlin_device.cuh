@@ -82,6 +82,17 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Programmatic dependent launch.  Kernels are launched with programmatic
+// stream serialization: the next kernel in the stream may start its
+// prologue while this one finishes.  grid_dep_wait() blocks until the
+// preceding kernel has completed and its memory operations are visible (a
+// no-op when launched without the attribute); every read or write of global
+// data comes after it.  grid_dep_launch() lets the next kernel begin.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // Shared abort state of one CTA: once any role's wait expires, every role
 // leaves its loop so the CTA can release TMEM and exit.
 struct WaitCtl {

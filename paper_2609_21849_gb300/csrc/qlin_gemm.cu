@@ -192,6 +192,9 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const WaitCtl ctl{abort_flag, p.err, p.timeout_ns};
+  // the prologue above overlaps the previous kernel; global data only below
+  grid_dep_wait();
+  grid_dep_launch();
 
   const int tiles_m = (int)((p.M + kBM - 1) / kBM);
   const int tiles_n = (int)((p.N + kBN - 1) / kBN);
@@ -730,16 +733,18 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   auto kern = gemm_kernel<kFp4, kBN, kPair, kRequant>;
 
   cudaLaunchConfig_t cfg{};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = kCM;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.blockDim = dim3(C::kThreads, 1, 1);
   cfg.dynamicSmemBytes = C::kSmemBytes;
   cfg.stream = s;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 1;   // the occupancy query below takes the cluster attribute only
 
   // one-time per instantiation: opt into the shared memory size and find how
   // many clusters fit at once (a persistent grid never exceeds that)
@@ -759,6 +764,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   const int64_t ctiles = ((tiles_m + kCM - 1) / kCM) * ((a.N + kBN - 1) / kBN);
   const int clusters = (int)std::min<int64_t>(ctiles, std::min(max_clusters, num_sms / kCM));
   cfg.gridDim = dim3((unsigned)(clusters * kCM), 1, 1);
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kern, ta, tb, tsa, tsb, ty, p);
 }
 

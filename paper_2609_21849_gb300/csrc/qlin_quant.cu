@@ -295,6 +295,8 @@ __device__ __forceinline__ bool stream_tiles(const uint4* __restrict__ x, uint64
 __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
     amax_kernel(const uint4* __restrict__ x, uint64_t n_chunks, unsigned* __restrict__ amax_bits,
                 unsigned* err, uint64_t timeout_ns) {
+  grid_dep_wait();
+  grid_dep_launch();
   __shared__ uint32_t warp_max[kThreads / 32];
   AmaxOp op;
   stream_tiles(x, n_chunks, op, err, timeout_ns);
@@ -330,6 +332,8 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
     quant_nvfp4_kernel(const uint4* __restrict__ x, uint64_t n_chunks, int64_t K,
                        const float* scale_src, float* sdec_out, uint32_t* __restrict__ codes,
                        uint8_t* __restrict__ scales, unsigned* err, uint64_t timeout_ns) {
+  grid_dep_wait();
+  grid_dep_launch();
   __shared__ float r_table[128];
   Nvfp4Op<Idx> op;
   op.r_table = r_table;
@@ -346,6 +350,8 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
     quant_fp8_kernel(const uint4* __restrict__ x, uint64_t n_chunks, const float* scale_src,
                      float* sdec_out, uint2* __restrict__ codes, unsigned* err,
                      uint64_t timeout_ns) {
+  grid_dep_wait();
+  grid_dep_launch();
   Fp8Op op;
   op.s_enc = encode_scale(tensor_scale<kDynamic>(scale_src, sdec_out, 448.0f));
   op.codes = codes;
@@ -358,6 +364,8 @@ __global__ void __launch_bounds__(kThreads) quant_fp8_rows_kernel(const uint4* _
                                                                   int64_t rows, int64_t K,
                                                                   float* __restrict__ s_rows,
                                                                   uint2* __restrict__ codes) {
+  grid_dep_wait();
+  grid_dep_launch();
   const int lane = threadIdx.x & 31;
   const int64_t cpr = K >> 3;
   const int64_t warp = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5;
@@ -416,6 +424,7 @@ __global__ void __launch_bounds__(kOnePassThreads, 1)
   __shared__ float op_table[128];
   __shared__ float s_amax;
   __shared__ int abort_flag;
+  grid_dep_wait();
   const int tid = threadIdx.x;
   const uint64_t c_begin = (uint64_t)blockIdx.x * slice;
   const uint32_t n = c_begin >= n_chunks ? 0u
@@ -425,6 +434,7 @@ __global__ void __launch_bounds__(kOnePassThreads, 1)
   const uint4* xs = x + c_begin;
   for (uint32_t i = tid; i < n; i += kOnePassThreads) cp_async16(smem_u32(buf + i), xs + i);
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
+  grid_dep_launch();   // x is on chip: the next kernel may begin launching
   uint32_t m = 0;
   for (uint32_t i = tid; i < n; i += kOnePassThreads) m = max(m, chunk_abs_max_bits(lds128(buf + i)));
   m = __reduce_max_sync(0xFFFFFFFFu, m);
@@ -469,6 +479,23 @@ cudaError_t set_smem() {
   return e;
 }
 
+// Launch with programmatic stream serialization (see grid_dep_wait).
+template <typename... Params, typename... Args>
+cudaError_t launch_pdl(void (*kern)(Params...), int grid, int block, int smem, cudaStream_t s,
+                       Args... args) {
+  cudaLaunchConfig_t cfg{};
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3((unsigned)grid, 1, 1);
+  cfg.blockDim = dim3((unsigned)block, 1, 1);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  cfg.stream = s;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 int stream_grid(uint64_t n_chunks, int num_sms) {
   const uint64_t tiles = (n_chunks + kTileChunks - 1) / kTileChunks;
   return (int)std::max<uint64_t>(1, std::min<uint64_t>(tiles, (uint64_t)num_sms * kBlocksPerSm));
@@ -482,9 +509,8 @@ cudaError_t launch_amax(const void* x, int64_t n_elems, unsigned* amax_bits, cud
   if (e != cudaSuccess) return e;
   if ((e = set_smem<amax_kernel>()) != cudaSuccess) return e;
   const uint64_t n_chunks = (uint64_t)n_elems / 8;
-  amax_kernel<<<stream_grid(n_chunks, num_sms), kThreads, kSmem, s>>>(
-      static_cast<const uint4*>(x), n_chunks, amax_bits, err, timeout_ns);
-  return cudaGetLastError();
+  return launch_pdl(amax_kernel, stream_grid(n_chunks, num_sms), kThreads, kSmem, s,
+                    static_cast<const uint4*>(x), n_chunks, amax_bits, err, timeout_ns);
 }
 
 // One-pass dynamic quantization when x fits on chip: returns
@@ -564,17 +590,15 @@ static cudaError_t launch_nvfp4_t(const void* x, int64_t M, int64_t K, const flo
   auto* codes = reinterpret_cast<uint32_t*>(out.codes);
   cudaError_t e;
   if (n_chunks < (1ull << 32)) {   // 32-bit index math is enough
-    auto kern = quant_nvfp4_kernel<kDynamic, uint32_t>;
     if ((e = set_smem<quant_nvfp4_kernel<kDynamic, uint32_t>>()) != cudaSuccess) return e;
-    kern<<<grid, kThreads, kSmem, s>>>(xin, n_chunks, K, scale_src, out.tensor_scale, codes,
-                                      out.scales, err, timeout_ns);
+    e = launch_pdl(quant_nvfp4_kernel<kDynamic, uint32_t>, grid, kThreads, kSmem, s, xin,
+                   n_chunks, K, scale_src, out.tensor_scale, codes, out.scales, err, timeout_ns);
   } else {
-    auto kern = quant_nvfp4_kernel<kDynamic, uint64_t>;
     if ((e = set_smem<quant_nvfp4_kernel<kDynamic, uint64_t>>()) != cudaSuccess) return e;
-    kern<<<grid, kThreads, kSmem, s>>>(xin, n_chunks, K, scale_src, out.tensor_scale, codes,
-                                      out.scales, err, timeout_ns);
+    e = launch_pdl(quant_nvfp4_kernel<kDynamic, uint64_t>, grid, kThreads, kSmem, s, xin,
+                   n_chunks, K, scale_src, out.tensor_scale, codes, out.scales, err, timeout_ns);
   }
-  return cudaGetLastError();
+  return e;
 }
 
 cudaError_t launch_quant_nvfp4(const void* x, int64_t M, int64_t K, const float* scale_src,
@@ -594,23 +618,20 @@ cudaError_t launch_quant_fp8(const void* x, int64_t M, int64_t K, const float* s
   cudaError_t e;
   if (dynamic) {
     if ((e = set_smem<quant_fp8_kernel<true>>()) != cudaSuccess) return e;
-    quant_fp8_kernel<true><<<grid, kThreads, kSmem, s>>>(xin, n_chunks, scale_src, out.scale,
-                                                         codes, err, timeout_ns);
-  } else {
-    if ((e = set_smem<quant_fp8_kernel<false>>()) != cudaSuccess) return e;
-    quant_fp8_kernel<false><<<grid, kThreads, kSmem, s>>>(xin, n_chunks, scale_src, out.scale,
-                                                          codes, err, timeout_ns);
+    return launch_pdl(quant_fp8_kernel<true>, grid, kThreads, kSmem, s, xin, n_chunks, scale_src,
+                      out.scale, codes, err, timeout_ns);
   }
-  return cudaGetLastError();
+  if ((e = set_smem<quant_fp8_kernel<false>>()) != cudaSuccess) return e;
+  return launch_pdl(quant_fp8_kernel<false>, grid, kThreads, kSmem, s, xin, n_chunks, scale_src,
+                    out.scale, codes, err, timeout_ns);
 }
 
 cudaError_t launch_quant_fp8_rows(const void* w, int64_t N, int64_t K, const qlin_fp8_t& out,
                                   cudaStream_t s, int num_sms) {
   const int64_t want = (N + kThreads / 32 - 1) / (kThreads / 32);
   const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)num_sms * 8));
-  quant_fp8_rows_kernel<<<grid, kThreads, 0, s>>>(static_cast<const uint4*>(w), N, K, out.scale,
-                                                  reinterpret_cast<uint2*>(out.codes));
-  return cudaGetLastError();
+  return launch_pdl(quant_fp8_rows_kernel, grid, kThreads, 0, s, static_cast<const uint4*>(w), N, K,
+                    out.scale, reinterpret_cast<uint2*>(out.codes));
 }
 
 }  // namespace qlin
