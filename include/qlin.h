@@ -117,8 +117,11 @@ size_t qlin_workspace_size(int64_t M, int64_t K);
  *  out:          rows == M, K == K; codes, scales and tensor_scale are written
  *                (tensor_scale receives S_dec in both modes).
  *  workspace:    device memory of >= qlin_workspace_size() bytes, 4-byte
- *                aligned; used (and overwritten) only in dynamic mode, may be
- *                NULL in static mode.
+ *                aligned, zero-filled before its first use; every call leaves
+ *                it zero-filled again (its words carry a grid-wide amax and
+ *                arrival counts inside one call).  Used only in dynamic mode,
+ *                may be NULL in static mode.  Calls whose work overlaps on
+ *                the GPU must not share one workspace.
  * Per 16-element block b (READING of the op order, each fp32 op rounded once):
  *   S_enc = 1 / S_dec (FLT_MAX if that overflows);
  *   s_b = E4M3((amax_b * S_enc) / 6);  r_b = s_b == 0 ? 0 : S_enc / s_b;
@@ -204,9 +207,9 @@ qlin_status qlin_linear_fused(const qlin_nvfp4_t *A, const qlin_nvfp4_t *W,
  * real-time loop that must never stall on cudaMalloc.  They can still pass x
  * and the output buffers, but not the workspace the dynamic amax pass needs.
  *
- * This entry point takes no workspace: its scratch (the amax word) lives in a
- * static device array of QLIN_NOALLOC_SCRATCH_BYTES bytes that the library
- * holds on every GPU that loads it, until the process exits.  It calls no
+ * This entry point takes no workspace: its scratch (the amax and arrival
+ * words) lives in a static device array of QLIN_NOALLOC_SCRATCH_BYTES bytes
+ * that the library holds on every GPU that loads it, until the process exits.  It calls no
  * cudaMalloc, cudaFree or other allocating routine.
  *  - x, M, K, out: as for qlin_quantize_act_nvfp4 (out->tensor_scale receives
  *    the dynamic S_dec = amax / 2688).

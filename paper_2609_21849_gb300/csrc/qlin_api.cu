@@ -117,15 +117,24 @@ qlin_status check_workspace(void* ws, size_t ws_bytes) {
   } while (0)
 
 }  // namespace
+// Workspace words of the dynamic tensor scale: the one-read route's amax,
+// arrival and departure counts (zero between calls), and the amax word of the
+// two-pass route (cleared before each use).
+constexpr int kWsOnePass = 0;
+constexpr int kWsTwoPassAmax = 4;
+
 // Dynamic NVFP4 activation quantization: one read of x when it fits on chip,
-// else the amax pass then the quantizer.  ws: at least two device words.
+// else the amax pass then the quantizer.  clear: zero the one-read words first.
 cudaError_t quant_nvfp4_dynamic(const void* x, int64_t M, int64_t K, const qlin_nvfp4_t& out,
-                                unsigned* ws, cudaStream_t s, int sms, unsigned* status) {
-  cudaError_t e = launch_quant_nvfp4_onepass(x, M, K, out, ws, s, sms, status, timeout());
+                                unsigned* ws, bool clear, cudaStream_t s, int sms,
+                                unsigned* status) {
+  cudaError_t e =
+      launch_quant_nvfp4_onepass(x, M, K, out, ws + kWsOnePass, clear, s, sms, status, timeout());
   if (e != cudaErrorNotSupported) return e;
-  if ((e = launch_amax(x, M * K, ws, s, sms, status, timeout())) != cudaSuccess) return e;
-  return launch_quant_nvfp4(x, M, K, reinterpret_cast<const float*>(ws), true, out, s, sms, status,
-                            timeout());
+  unsigned* amax = ws + kWsTwoPassAmax;
+  if ((e = launch_amax(x, M * K, amax, s, sms, status, timeout())) != cudaSuccess) return e;
+  return launch_quant_nvfp4(x, M, K, reinterpret_cast<const float*>(amax), true, out, s, sms,
+                            status, timeout());
 }
 
 }  // namespace qlin
@@ -158,8 +167,8 @@ qlin_status qlin_quantize_act_nvfp4(const void* x_bf16, int64_t M, int64_t K,
   QLIN_TRY(device_state(&status, &sms));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (static_scale == nullptr) {
-    QLIN_CUDA(quant_nvfp4_dynamic(x_bf16, M, K, *out, static_cast<unsigned*>(workspace), s, sms,
-                                  status));
+    QLIN_CUDA(quant_nvfp4_dynamic(x_bf16, M, K, *out, static_cast<unsigned*>(workspace), false, s,
+                                  sms, status));
   } else {
     QLIN_CUDA(launch_quant_nvfp4(x_bf16, M, K, static_scale, false, *out, s, sms, status, timeout()));
   }
@@ -184,8 +193,8 @@ qlin_status qlin_quantize_act_nvfp4_noalloc(const void* x_bf16, int64_t M, int64
   QLIN_TRY(noalloc_scratch(&scratch));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // the scratch words are cleared by the launch that uses them
-  QLIN_CUDA(quant_nvfp4_dynamic(x_bf16, M, K, *out, reinterpret_cast<unsigned*>(scratch), s, sms,
-                                status));
+  QLIN_CUDA(quant_nvfp4_dynamic(x_bf16, M, K, *out, reinterpret_cast<unsigned*>(scratch), true, s,
+                                sms, status));
   return QLIN_OK;
 }
 
@@ -204,10 +213,12 @@ qlin_status qlin_quantize_act_fp8(const void* x_bf16, int64_t M, int64_t K,
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (static_scale == nullptr) {
     unsigned* ws = static_cast<unsigned*>(workspace);
-    cudaError_t e = launch_quant_fp8_onepass(x_bf16, M, K, *out, ws, s, sms, status, timeout());
+    cudaError_t e = launch_quant_fp8_onepass(x_bf16, M, K, *out, ws + kWsOnePass, false, s, sms,
+                                             status, timeout());
     if (e == cudaErrorNotSupported) {   // x does not fit on chip: amax pass, then quantize
-      QLIN_CUDA(launch_amax(x_bf16, M * K, ws, s, sms, status, timeout()));
-      e = launch_quant_fp8(x_bf16, M, K, reinterpret_cast<const float*>(ws), true, *out, s, sms,
+      unsigned* amax = ws + kWsTwoPassAmax;
+      QLIN_CUDA(launch_amax(x_bf16, M * K, amax, s, sms, status, timeout()));
+      e = launch_quant_fp8(x_bf16, M, K, reinterpret_cast<const float*>(amax), true, *out, s, sms,
                            status, timeout());
     }
     QLIN_CUDA(e);

@@ -23,14 +23,17 @@ cudaError_t launch_quant_fp8(const void* x, int64_t M, int64_t K, const float* s
                              bool dynamic, const qlin_fp8_t& out, cudaStream_t s, int num_sms,
                              unsigned* err, uint64_t timeout_ns);
 // Dynamic tensor scale in one read of x (x held on chip across the grid).
-// sync: two device words of scratch.  Returns cudaErrorNotSupported, having
-// launched nothing, when x does not fit; the caller then runs amax + quant.
+// sync: three device words of scratch, zero at launch (clear = zero them
+// first) and zero again when the kernel ends.  Returns cudaErrorNotSupported,
+// having launched nothing, when x does not fit; the caller then runs amax +
+// quant.
 cudaError_t launch_quant_nvfp4_onepass(const void* x, int64_t M, int64_t K,
-                                       const qlin_nvfp4_t& out, unsigned* sync, cudaStream_t s,
-                                       int num_sms, unsigned* err, uint64_t timeout_ns);
+                                       const qlin_nvfp4_t& out, unsigned* sync, bool clear,
+                                       cudaStream_t s, int num_sms, unsigned* err,
+                                       uint64_t timeout_ns);
 cudaError_t launch_quant_fp8_onepass(const void* x, int64_t M, int64_t K, const qlin_fp8_t& out,
-                                     unsigned* sync, cudaStream_t s, int num_sms, unsigned* err,
-                                     uint64_t timeout_ns);
+                                     unsigned* sync, bool clear, cudaStream_t s, int num_sms,
+                                     unsigned* err, uint64_t timeout_ns);
 cudaError_t launch_quant_fp8_rows(const void* w, int64_t N, int64_t K, const qlin_fp8_t& out,
                                   cudaStream_t s, int num_sms);
 

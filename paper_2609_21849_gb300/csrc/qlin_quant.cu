@@ -407,12 +407,13 @@ __device__ __forceinline__ uint32_t ld_acquire_gpu(const unsigned* p) {
   return v;
 }
 
-// sync[0]: amax bits (fp32), sync[1]: arrival count; both zero at launch.
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
 }
 
-// sync[0]: amax bits (fp32), sync[1]: arrival count; both zero at launch.
+// sync[0]: amax bits (fp32), sync[1]: arrival count, sync[2]: departure
+// count; all zero at launch, and the last CTA to depart zeroes them again, so
+// back-to-back launches (graph replays included) need no clearing between.
 template <typename Op>
 __global__ void __launch_bounds__(kOnePassThreads, 1)
     onepass_kernel(const uint4* __restrict__ x, uint64_t n_chunks, uint32_t slice, Op op,
@@ -458,6 +459,12 @@ __global__ void __launch_bounds__(kOnePassThreads, 1)
       }
     }
     s_amax = __uint_as_float(ld_acquire_gpu(&sync[0]));
+    // depart (after a timeout too); the last CTA out resets the words
+    if (atomicAdd(&sync[2], 1u) == gridDim.x - 1u) {
+      sync[0] = 0u;
+      sync[1] = 0u;
+      sync[2] = 0u;
+    }
   }
   __syncthreads();
   if (abort_flag) return;
@@ -518,8 +525,8 @@ cudaError_t launch_amax(const void* x, int64_t n_elems, unsigned* amax_bits, cud
 // device cannot hold the grid resident.
 template <typename Op>
 static cudaError_t launch_onepass(const void* x, uint64_t n_chunks, const Op& op, float qmax,
-                                  float* sdec_out, unsigned* sync, cudaStream_t s, int num_sms,
-                                  unsigned* err, uint64_t timeout_ns) {
+                                  float* sdec_out, unsigned* sync, bool clear, cudaStream_t s,
+                                  int num_sms, unsigned* err, uint64_t timeout_ns) {
   // slices of whole 64-element groups (8 chunks), one per SM
   uint64_t slice = (n_chunks + num_sms - 1) / num_sms;
   slice = (slice + 7) / 8 * 8;
@@ -538,25 +545,41 @@ static cudaError_t launch_onepass(const void* x, uint64_t n_chunks, const Op& op
     resident = r;
   }
   if (resident < 1 || grid > num_sms * resident) return cudaErrorNotSupported;
-  cudaError_t e = cudaMemsetAsync(sync, 0, 2 * sizeof(unsigned), s);
-  if (e != cudaSuccess) return e;
+  if (clear) {
+    const cudaError_t e = cudaMemsetAsync(sync, 0, 3 * sizeof(unsigned), s);
+    if (e != cudaSuccess) return e;
+  }
   cudaLaunchConfig_t cfg{};
-  cudaLaunchAttribute at[1];
+  cudaLaunchAttribute at[2];
   at[0].id = cudaLaunchAttributeCooperative;   // all CTAs resident: the grid waits on itself
   at[0].val.cooperative = 1;
+  at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3((unsigned)grid, 1, 1);
   cfg.blockDim = dim3(kOnePassThreads, 1, 1);
   cfg.dynamicSmemBytes = kOnePassSmem;
   cfg.stream = s;
   cfg.attrs = at;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, static_cast<const uint4*>(x), n_chunks, (uint32_t)slice,
-                            op, qmax, sdec_out, sync, err, timeout_ns);
+  // with programmatic serialization where the driver accepts it alongside a
+  // cooperative launch, else without
+  static bool pdl_ok = true;
+  cfg.numAttrs = pdl_ok ? 2 : 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kern, static_cast<const uint4*>(x), n_chunks,
+                                     (uint32_t)slice, op, qmax, sdec_out, sync, err, timeout_ns);
+  if (e != cudaSuccess && pdl_ok) {
+    (void)cudaGetLastError();
+    pdl_ok = false;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kern, static_cast<const uint4*>(x), n_chunks, (uint32_t)slice,
+                           op, qmax, sdec_out, sync, err, timeout_ns);
+  }
+  return e;
 }
 
 cudaError_t launch_quant_nvfp4_onepass(const void* x, int64_t M, int64_t K,
-                                       const qlin_nvfp4_t& out, unsigned* sync, cudaStream_t s,
-                                       int num_sms, unsigned* err, uint64_t timeout_ns) {
+                                       const qlin_nvfp4_t& out, unsigned* sync, bool clear,
+                                       cudaStream_t s, int num_sms, unsigned* err,
+                                       uint64_t timeout_ns) {
   const uint64_t n_chunks = (uint64_t)M * (uint64_t)K / 8;
   if (n_chunks >= (1ull << 32)) return cudaErrorNotSupported;
   Nvfp4Op<uint32_t> op;
@@ -566,18 +589,19 @@ cudaError_t launch_quant_nvfp4_onepass(const void* x, int64_t M, int64_t K,
   op.codes = reinterpret_cast<uint32_t*>(out.codes);
   op.scales = out.scales;
   op.r_table = nullptr;   // set in the kernel (shared memory)
-  return launch_onepass(x, n_chunks, op, 2688.0f, out.tensor_scale, sync, s, num_sms, err,
+  return launch_onepass(x, n_chunks, op, 2688.0f, out.tensor_scale, sync, clear, s, num_sms, err,
                         timeout_ns);
 }
 
 cudaError_t launch_quant_fp8_onepass(const void* x, int64_t M, int64_t K, const qlin_fp8_t& out,
-                                     unsigned* sync, cudaStream_t s, int num_sms, unsigned* err,
-                                     uint64_t timeout_ns) {
+                                     unsigned* sync, bool clear, cudaStream_t s, int num_sms,
+                                     unsigned* err, uint64_t timeout_ns) {
   const uint64_t n_chunks = (uint64_t)M * (uint64_t)K / 8;
   Fp8Op op;
   op.s_enc = 0.0f;
   op.codes = reinterpret_cast<uint2*>(out.codes);
-  return launch_onepass(x, n_chunks, op, 448.0f, out.scale, sync, s, num_sms, err, timeout_ns);
+  return launch_onepass(x, n_chunks, op, 448.0f, out.scale, sync, clear, s, num_sms, err,
+                        timeout_ns);
 }
 
 template <bool kDynamic>

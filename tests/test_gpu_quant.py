@@ -160,3 +160,18 @@ def test_dynamic_scale_one_read_repeated():
         q = qlin.qlin_quantize_act_nvfp4(to_dev(xb), None, qlin.alloc_nvfp4(M, K), ws)
         assert qlin.qlin_sync_status() == 0
         assert_nvfp4_equal(q, oracle.quant_nvfp4(xb), f"gain {gain}")
+
+
+def test_dynamic_scale_workspace_shared_by_both_routes():
+    # one workspace serves the one-read route (words left zero after each
+    # call) and the two-pass route (its own amax word, cleared before use):
+    # alternate them and each must still equal the oracle
+    ws = qlin.alloc_workspace()
+    small = synthetic.act_entry_outliers(31, 512, 1024)     # fits on chip
+    large = synthetic.act_normal(32, 9216, 4096)            # does not
+    for x in (large, small, large, small):
+        M, K = x.shape
+        q = qlin.qlin_quantize_act_nvfp4(to_dev(x), None, qlin.alloc_nvfp4(M, K), ws)
+        assert qlin.qlin_sync_status() == 0
+        assert_nvfp4_equal(q, oracle.quant_nvfp4(x), f"{M}x{K}")
+    assert int(ws[:12].sum()) == 0   # the one-read words are left zeroed
