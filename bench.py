@@ -256,24 +256,62 @@ def run_ours(args, dist: Dist):
                        200, torch, stream)
     gemm_tflops = STEP_FLOPS / gemm_s / 1e12
 
-    # ---- end to end through the public API with host buffers
+    # ---- end to end through the public API with host buffers: every step
+    # copies its x in from pinned host memory and its y out to pinned host
+    # memory inside the timed region.  The copies run on streams of their own,
+    # so one step's compute overlaps the next step's input copy and the
+    # previous step's output copy, as a serving loop does; events keep each
+    # step's copy-in -> compute -> copy-out order and each set's reuse order.
     x_host = torch.from_numpy(x_bits.view(np.int16)).pin_memory()
-    y_host = torch.empty((M, N), dtype=torch.int16).pin_memory()
+    y_hosts = [torch.empty((M, N), dtype=torch.int16).pin_memory() for _ in range(R)]
+    # (the output copy, 113 MB, runs at ~190 GB/s device -> host; splitting it
+    # over several streams measured no faster)
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    ev_in = [torch.cuda.Event() for _ in range(R)]
+    ev_comp = [torch.cuda.Event() for _ in range(R)]
+    ev_out = [torch.cuda.Event() for _ in range(R)]
 
-    def e2e_step(r):
-        xs[r].view(torch.int16).copy_(x_host, non_blocking=True)
-        step(r)
-        y_host.copy_(ys[r].view(torch.int16), non_blocking=True)
+    def e2e_step(i):
+        r = i % R
+        s_in.wait_event(ev_comp[r])             # the set's last compute has read xs[r]
+        with torch.cuda.stream(s_in):
+            xs[r].view(torch.int16).copy_(x_host, non_blocking=True)
+        ev_in[r].record(s_in)
+        stream.wait_event(ev_in[r])
+        stream.wait_event(ev_out[r])            # the set's last output has been read
+        with torch.cuda.stream(stream):
+            step(r)
+        ev_comp[r].record(stream)
+        s_out.wait_event(ev_comp[r])
+        with torch.cuda.stream(s_out):
+            y_hosts[r].copy_(ys[r].view(torch.int16), non_blocking=True)
+        ev_out[r].record(s_out)
 
-    for r in range(R):
-        e2e_step(r)
-    n_e2e = max(R, min(200, steps // 10))
-    e2e_sec = timed(lambda c=[0]: (e2e_step(c[0] % R), c.__setitem__(0, c[0] + 1)), n_e2e, torch,
-                    stream)
-    e2e_sec = dist.max(e2e_sec)
+    def e2e_run(n):
+        torch.cuda.synchronize()
+        for r in range(R):
+            ev_comp[r].record(stream)
+            ev_out[r].record(stream)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        s_in.wait_event(a)
+        s_out.wait_event(a)
+        for i in range(n):
+            e2e_step(i)
+        for r in range(R):
+            stream.wait_event(ev_out[r])
+        b.record(stream)
+        b.synchronize()
+        return a.elapsed_time(b) / 1e3 / n
+
+    e2e_run(2 * R)                              # warm-up
+    n_e2e = max(4 * R, min(200, steps // 10))
+    e2e_sec = dist.max(e2e_run(n_e2e))
     e2e = {"value": round(STEP_FLOPS * dist.world / e2e_sec / 1e12, 2), "unit": "TFLOP/s",
            "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2,
-           "ms_per_step": round(e2e_sec * 1e3, 4)}
+           "ms_per_step": round(e2e_sec * 1e3, 4),
+           "copies": "pinned host buffers; input copy, compute and output copy on three "
+                     "streams, consecutive steps overlapped"}
 
     traffic = committed_traffic()
     out = {
@@ -283,11 +321,11 @@ def run_ours(args, dist: Dist):
         "scaling": "weak", "vs_baseline": None, "dtype": "nvfp4 (e2m1 x e4m3 block scales), fp32 accumulate, bf16 out",
         "data": "synthetic (seeded; shapes of FLUX.2-klein at 1024^2, random weights)",
         "config": {"workload": WORKLOAD, "M": M, "N": N, "K": K,
-                   "step": "dynamic NVFP4 act quant (amax+quant) + NVFP4 GEMM + bf16 out + fused NVFP4 requant",
+                   "step": "dynamic NVFP4 act quant (one read of x: grid-wide amax + quant) + NVFP4 GEMM + bf16 out + fused NVFP4 requant",
                    "l2": f"{R} rotating input/output sets of {set_bytes / 2**20:.0f} MiB each (> 129 MiB L2)",
                    "graph": f"CUDA graph of {S} steps replayed {replays}x",
                    "parallelism": f"replicas x{dist.world}"},
-        "gpu_launches": 3 * steps,
+        "gpu_launches": 2 * steps,
         "clocks": clk,
         "e2e": e2e,
         "roofline": {"kernel": "gemm_kernel<nvfp4, BN=256, requant>", "bound": "tensor",
