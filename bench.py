@@ -432,7 +432,15 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
     t = g_time(lambda: (lambda r: qlin.qlin_gemm_nvfp4(A4[r % 2], W4[r % 2], y4[r % 2]))(nxt()), 4)
     rows["a5_gemm_nvfp4"] = {"us": round(t * 1e6, 2), "TFLOP/s": round(STEP_FLOPS / t / 1e12, 1),
                              "frac_fp4_peak": round(STEP_FLOPS / t / 1e12 / fp4_peak, 3)}
-    del A4, W4, y4
+    # the same linear with the next layer's input quantized at y's own dynamic
+    # scale (epilogue amax + a quantizer pass over y: 113 MB read, 35 MB written)
+    yq4 = [qlin.alloc_nvfp4(M, N) for _ in range(2)]
+    wsd = [qlin.alloc_workspace() for _ in range(2)]
+    t = g_time(lambda: (lambda r: qlin.qlin_linear_dynamic(A4[r % 2], W4[r % 2], y4[r % 2], yq4[r % 2],
+                                                           wsd[r % 2]))(nxt()), 4)
+    rows["f1_linear_dynamic_nvfp4"] = {"us": round(t * 1e6, 2), "TFLOP/s": round(STEP_FLOPS / t / 1e12, 1),
+                                       "note": "GEMM with output-amax epilogue + NVFP4 quantizer over y"}
+    del A4, W4, y4, yq4
 
     # small-M translator linears (batch 1, 512 tokens), both formats, latency
     x1, x2, w1, w2 = synthetic.translator()

@@ -227,6 +227,28 @@ qlin_status qlin_quantize_act_nvfp4_noalloc(const void *x_bf16, int64_t M, int64
                                             qlin_nvfp4_t *out, void *stream);
 
 /*
+ * Dynamic per-tensor scaling inside a chain of linears (Sec. 4, "Quantization":
+ * run-time activation quantization, here with the tensor scale of the layer's
+ * own output instead of a calibrated one):
+ *   y = A W^T (bf16, as qlin_gemm_nvfp4), while the GEMM epilogue reduces
+ *   amax(|y|) into a workspace word; then y_q = NVFP4(y) with the dynamic
+ *   S_dec = amax / 2688 (1 if amax == 0), exactly as
+ *   qlin_quantize_act_nvfp4(y, NULL) would produce it, without its amax pass
+ *   over y.
+ *  A, W:      NVFP4 operands as for qlin_gemm_nvfp4.
+ *  y_bf16:    bf16 [A->rows, W->rows], 16-byte aligned (required: the
+ *             quantizer reads it).
+ *  y_q:       rows == A->rows, K == W->rows; codes, scales and tensor_scale
+ *             are written.
+ *  workspace: as for qlin_quantize_act_nvfp4 (one word of it is cleared and
+ *             used per call).
+ * Errors: INVALID_ARG, MISALIGNED, WORKSPACE, CUDA.
+ */
+qlin_status qlin_linear_dynamic(const qlin_nvfp4_t *A, const qlin_nvfp4_t *W, void *y_bf16,
+                                qlin_nvfp4_t *y_q, void *workspace, size_t ws_bytes,
+                                void *stream);
+
+/*
  * Waits for `stream`, then returns and clears the device status word:
  * QLIN_ERR_TIMEOUT if a kernel's bounded wait expired since the last call,
  * QLIN_ERR_CUDA if the stream reports an error, else QLIN_OK.

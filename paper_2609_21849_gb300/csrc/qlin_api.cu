@@ -122,6 +122,7 @@ qlin_status check_workspace(void* ws, size_t ws_bytes) {
 // two-pass route (cleared before each use).
 constexpr int kWsOnePass = 0;
 constexpr int kWsTwoPassAmax = 4;
+constexpr int kWsChainAmax = 5;   // qlin_linear_dynamic: max |y| from the GEMM epilogue
 
 // Dynamic NVFP4 activation quantization: one read of x when it fits on chip,
 // else the amax pass then the quantizer.  clear: zero the one-read words first.
@@ -249,8 +250,9 @@ qlin_status qlin_quantize_weight(const void* w_bf16, int64_t N, int64_t K, qlin_
 
 static qlin_status gemm_common(bool fp4, const void* Aany, const void* Wany, void* y,
                                const float* next_scale, qlin_nvfp4_t* y_q, int64_t rq_col0,
-                               void* stream) {
+                               void* stream, unsigned* y_amax = nullptr) {
   GemmArgs a{};
+  a.y_amax = y_amax;
   a.fp4 = fp4;
   if (fp4) {
     const qlin_nvfp4_t* A = static_cast<const qlin_nvfp4_t*>(Aany);
@@ -305,6 +307,8 @@ static qlin_status gemm_common(bool fp4, const void* Aany, const void* Wany, voi
   unsigned* status;
   int sms;
   QLIN_TRY(device_state(&status, &sms));
+  if (y_amax != nullptr)
+    QLIN_CUDA(cudaMemsetAsync(y_amax, 0, sizeof(unsigned), static_cast<cudaStream_t>(stream)));
   cudaError_t e = launch_gemm(a, static_cast<cudaStream_t>(stream), sms, status,
                               g_timeout_ns.load(std::memory_order_relaxed));
   if (e != cudaSuccess) return cuda_fail(e);
@@ -326,6 +330,26 @@ qlin_status qlin_linear_fused(const qlin_nvfp4_t* A, const qlin_nvfp4_t* W, void
                               const float* next_scale, qlin_nvfp4_t* y_q, int64_t rq_col0,
                               void* stream) {
   return gemm_common(true, A, W, y_bf16, next_scale, y_q, rq_col0, stream);
+}
+
+qlin_status qlin_linear_dynamic(const qlin_nvfp4_t* A, const qlin_nvfp4_t* W, void* y_bf16,
+                                qlin_nvfp4_t* y_q, void* workspace, size_t ws_bytes,
+                                void* stream) {
+  if (A == nullptr || W == nullptr || y_bf16 == nullptr || y_q == nullptr)
+    return QLIN_ERR_INVALID_ARG;
+  QLIN_TRY(check_nvfp4(y_q, A->rows, W->rows));
+  QLIN_TRY(check_workspace(workspace, ws_bytes));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unsigned* amax = static_cast<unsigned*>(workspace) + kWsChainAmax;
+  // y and its tensor amax in one GEMM (the word is cleared first), then the
+  // quantizer with that scale
+  QLIN_TRY(gemm_common(true, A, W, y_bf16, nullptr, nullptr, 0, stream, amax));
+  unsigned* status;
+  int sms;
+  QLIN_TRY(device_state(&status, &sms));
+  QLIN_CUDA(launch_quant_nvfp4(y_bf16, A->rows, W->rows, reinterpret_cast<const float*>(amax),
+                               true, *y_q, s, sms, status, timeout()));
+  return QLIN_OK;
 }
 
 qlin_status qlin_sync_status(void* stream) {

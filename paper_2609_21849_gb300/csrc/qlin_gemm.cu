@@ -105,6 +105,7 @@ struct KParams {
   uint8_t* rq_scales;
   float* rq_tensor_scale;
   int64_t rq_col0, rq_cols;
+  unsigned* y_amax;   // optional: max |bf16 y| over the output, as fp32 bits (atomicMax)
   unsigned* err;
   uint64_t timeout_ns;
 };
@@ -535,6 +536,18 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
         }
       }
 
+      if (p.y_amax != nullptr) {
+        // the output's tensor amax (for a dynamic scale of the next layer's
+        // input): max over this thread's bf16 values, then the warp, then
+        // one atomic per warp.  Rows past M and columns past N hold zeros
+        // (zero-filled operands), which leave the maximum unchanged.
+        uint32_t m = 0;
+#pragma unroll
+        for (int i = 0; i < kCols / 2; ++i) m = __vmaxu2(m, packed[i] & 0x7FFF7FFFu);
+        m = max(m & 0xFFFFu, m >> 16);
+        m = __reduce_max_sync(0xFFFFFFFFu, m);
+        if (lane == 0 && m != 0u) atomicMax(p.y_amax, m << 16);
+      }
       if (p.y != nullptr) {
         // bf16 output: each 32 x 32 box goes through a 64-byte-swizzled
         // staging buffer and one TMA store (rows >= M, cols >= N are clipped).
@@ -728,6 +741,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   p.rq_tensor_scale = a.rq_tensor_scale;
   p.rq_col0 = a.rq_col0;
   p.rq_cols = a.rq_cols;
+  p.y_amax = a.y_amax;
   p.err = err;
   p.timeout_ns = timeout_ns;
   auto kern = gemm_kernel<kFp4, kBN, kPair, kRequant>;

@@ -55,6 +55,8 @@ struct GemmArgs {
   uint8_t* rq_scales;
   float* rq_tensor_scale;
   int64_t rq_col0, rq_cols;
+  // optional max |bf16 y| (fp32 bits, atomicMax; cleared by the caller)
+  unsigned* y_amax;
 };
 cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned* err,
                         uint64_t timeout_ns);

@@ -24,7 +24,8 @@ STATUS = {0: "QLIN_OK", 1: "QLIN_ERR_INVALID_ARG", 2: "QLIN_ERR_UNSUPPORTED",
 # Every function declared in include/qlin.h.
 EXPORTS = ("qlin_nvfp4_scale_bytes", "qlin_workspace_size", "qlin_quantize_act_nvfp4",
            "qlin_quantize_act_fp8", "qlin_quantize_weight", "qlin_gemm_nvfp4", "qlin_gemm_fp8",
-           "qlin_linear_fused", "qlin_quantize_act_nvfp4_noalloc", "qlin_sync_status", "qlin_selftest_bounded_wait",
+           "qlin_linear_fused", "qlin_linear_dynamic", "qlin_quantize_act_nvfp4_noalloc",
+           "qlin_sync_status", "qlin_selftest_bounded_wait",
            "qlin_set_wait_timeout_ns", "qlin_status_str", "qlin_last_error")
 
 
@@ -71,6 +72,8 @@ def load_library(path: str = LIB_PATH):
             "qlin_gemm_fp8": (ctypes.c_int, [ctypes.POINTER(FP8Desc), ctypes.POINTER(FP8Desc), p, p]),
             "qlin_linear_fused": (ctypes.c_int, [ctypes.POINTER(NVFP4Desc), ctypes.POINTER(NVFP4Desc), p, p,
                                                  ctypes.POINTER(NVFP4Desc), i64, p]),
+            "qlin_linear_dynamic": (ctypes.c_int, [ctypes.POINTER(NVFP4Desc), ctypes.POINTER(NVFP4Desc), p,
+                                                   ctypes.POINTER(NVFP4Desc), p, sz, p]),
             "qlin_quantize_act_nvfp4_noalloc": (ctypes.c_int, [p, i64, i64, ctypes.POINTER(NVFP4Desc), p]),
             "qlin_sync_status": (ctypes.c_int, [p]),
             "qlin_selftest_bounded_wait": (ctypes.c_int, [ctypes.c_uint64, p]),
@@ -270,6 +273,25 @@ def qlin_linear_fused(A: NVFP4Tensor, W: NVFP4Tensor, y: torch.Tensor | None,
         ctypes.byref(da), ctypes.byref(dw), _ptr(y), _ptr(next_scale),
         ctypes.byref(dq) if dq is not None else None, rq_col0, _stream(stream)),
         "qlin_linear_fused")
+    return y, y_q
+
+
+def qlin_linear_dynamic(A: NVFP4Tensor, W: NVFP4Tensor, y: torch.Tensor | None = None,
+                        y_q: NVFP4Tensor | None = None, workspace: torch.Tensor | None = None,
+                        stream=None):
+    """y = A W^T (bf16) and y_q = NVFP4(y) with y's own dynamic tensor scale,
+    the amax taken in the GEMM epilogue.  Returns (y, y_q)."""
+    M, N = A.rows, W.rows
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.bfloat16, device=A.codes.device)
+    if y_q is None:
+        y_q = alloc_nvfp4(M, N, A.codes.device)
+    if workspace is None:
+        workspace = alloc_workspace(A.codes.device)
+    da, dw, dq = A.desc(), W.desc(), y_q.desc()
+    _check(load_library().qlin_linear_dynamic(
+        ctypes.byref(da), ctypes.byref(dw), _ptr(y), ctypes.byref(dq), _ptr(workspace),
+        workspace.numel(), _stream(stream)), "qlin_linear_dynamic")
     return y, y_q
 
 

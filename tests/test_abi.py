@@ -71,6 +71,15 @@ def test_argument_errors_return_before_launch(lib):
     q = qlin.NVFP4Desc(16, 16, 16, 128, 128)
     assert lib.qlin_linear_fused(ctypes.byref(a), ctypes.byref(w), 16, 16, ctypes.byref(q), 192,
                                  None) == 1
+    # dynamic chain: output descriptor of the wrong shape, missing workspace
+    q = qlin.NVFP4Desc(16, 16, 16, 128, 128)
+    assert lib.qlin_linear_dynamic(ctypes.byref(a), ctypes.byref(w), 16, ctypes.byref(q), 16, 256,
+                                   None) == 1
+    q = qlin.NVFP4Desc(16, 16, 16, 128, 256)
+    assert lib.qlin_linear_dynamic(ctypes.byref(a), ctypes.byref(w), 16, ctypes.byref(q), None, 0,
+                                   None) == 6
+    assert lib.qlin_linear_dynamic(ctypes.byref(a), ctypes.byref(w), None, ctypes.byref(q), 16, 256,
+                                   None) == 1
     # FP8: per-channel activation descriptor is rejected; unknown weight format
     f = qlin.FP8Desc(16, 16, 128, 256, 1)
     assert lib.qlin_quantize_act_fp8(16, 128, 256, 16, ctypes.byref(f), None, 0, None) == 1
