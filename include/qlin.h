@@ -227,6 +227,20 @@ qlin_status qlin_quantize_act_nvfp4_noalloc(const void *x_bf16, int64_t M, int64
                                             qlin_nvfp4_t *out, void *stream);
 
 /*
+ * Unquantized bf16 linear on the same tensor-core skeleton (tcgen05
+ * kind::f16), the reference precision of Table 2 (BF16 / FP8 / NVFP4 step
+ * latencies): y = a w^T, fp32 accumulation, bf16 out.
+ *  a_bf16: bf16 [M, K] with row stride lda (elements, lda >= K, lda * 2 a
+ *          multiple of 16), 16-byte aligned.  A strided view serves, e.g. the
+ *          value columns of a QKV output.
+ *  w_bf16: bf16 [N, K] row-major; y_bf16: bf16 [M, N].
+ *  K % 64 == 0, N % 64 == 0.
+ * Errors: INVALID_ARG, MISALIGNED, UNSUPPORTED, CUDA.
+ */
+qlin_status qlin_gemm_bf16(const void *a_bf16, int64_t lda, const void *w_bf16, int64_t M,
+                           int64_t N, int64_t K, void *y_bf16, void *stream);
+
+/*
  * Dynamic per-tensor scaling inside a chain of linears (Sec. 4, "Quantization":
  * run-time activation quantization, here with the tensor scale of the layer's
  * own output instead of a calibrated one):

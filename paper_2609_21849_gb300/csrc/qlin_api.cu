@@ -332,6 +332,31 @@ qlin_status qlin_linear_fused(const qlin_nvfp4_t* A, const qlin_nvfp4_t* W, void
   return gemm_common(true, A, W, y_bf16, next_scale, y_q, rq_col0, stream);
 }
 
+qlin_status qlin_gemm_bf16(const void* a_bf16, int64_t lda, const void* w_bf16, int64_t M,
+                           int64_t N, int64_t K, void* y_bf16, void* stream) {
+  if (a_bf16 == nullptr || w_bf16 == nullptr || y_bf16 == nullptr) return QLIN_ERR_INVALID_ARG;
+  if (M < 1 || K < 64 || K % 64 != 0 || N < 64 || N % 64 != 0 || lda < K)
+    return QLIN_ERR_INVALID_ARG;
+  if (M > (int64_t)1 << 31 || N > (int64_t)1 << 31) return QLIN_ERR_UNSUPPORTED;
+  if (!aligned(a_bf16, 16) || !aligned(w_bf16, 16) || !aligned(y_bf16, 16) || (lda * 2) % 16 != 0)
+    return QLIN_ERR_MISALIGNED;
+  GemmArgs a{};
+  a.bf16 = true;
+  a.a_codes = a_bf16;
+  a.a_row_bytes = lda * 2;
+  a.w_codes = w_bf16;
+  a.y = y_bf16;
+  a.M = M;
+  a.N = N;
+  a.K = K;
+  unsigned* status;
+  int sms;
+  QLIN_TRY(device_state(&status, &sms));
+  cudaError_t e = launch_gemm(a, static_cast<cudaStream_t>(stream), sms, status, timeout());
+  if (e != cudaSuccess) return cuda_fail(e);
+  return QLIN_OK;
+}
+
 qlin_status qlin_linear_dynamic(const qlin_nvfp4_t* A, const qlin_nvfp4_t* W, void* y_bf16,
                                 qlin_nvfp4_t* y_q, void* workspace, size_t ws_bytes,
                                 void* stream) {

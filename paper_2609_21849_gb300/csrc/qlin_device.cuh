@@ -359,6 +359,17 @@ __device__ __forceinline__ void mma_fp8_pair(uint32_t d_tmem, uint64_t a_desc, u
       : "memory");
 }
 
+// Same, bf16 operands (kind::f16), K = 16 per instruction.
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                              uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // Address of the same shared-memory variable in CTA `rank` of the cluster.
 __device__ __forceinline__ uint32_t mapa_shared(const void* p, uint32_t rank) {
   uint32_t r;
@@ -431,6 +442,16 @@ __device__ __forceinline__ void mma_fp8(uint32_t d_tmem, uint64_t a_desc, uint64
       : "memory");
 }
 
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // Instruction descriptor, block-scaled NVFP4 (kind::mxf4nvf4): e2m1 A and B,
 // both K-major, UE4M3 scales, M = 128, N = n.
 __host__ __device__ constexpr uint32_t idesc_nvfp4(int n, int m = 128) {
@@ -445,6 +466,13 @@ __host__ __device__ constexpr uint32_t idesc_nvfp4(int n, int m = 128) {
 __host__ __device__ constexpr uint32_t idesc_fp8(int n, int m = 128) {
   return (1u << 4)                      // D format: f32
          | (0u << 7) | (0u << 10)       // A, B: E4M3
+         | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+// Instruction descriptor, kind::f16: bf16 A and B (K-major), fp32 accumulator.
+__host__ __device__ constexpr uint32_t idesc_bf16(int n, int m = 128) {
+  return (1u << 4)                      // D format: f32
+         | (1u << 7) | (1u << 10)       // A, B: bf16
          | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 

@@ -131,7 +131,9 @@ __device__ __forceinline__ void st_global_v4(void* p, uint32_t a, uint32_t b, ui
                : "memory");
 }
 
-template <bool kFp4, int kBN, bool kPair, bool kRequant>
+// kBf16 (with !kFp4): bf16 operands on the FP8 skeleton (the same 128-byte
+// rows, 32 bytes of K per MMA), no scales.
+template <bool kFp4, int kBN, bool kPair, bool kRequant, bool kBf16 = false>
 __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_a,
                 const __grid_constant__ CUtensorMap tmap_b,
@@ -203,7 +205,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
   const int num_ctiles = groups_m * tiles_n;
   const int cid = (int)blockIdx.x / kCM;
   const int ncl = (int)gridDim.x / kCM;
-  const int64_t k_bytes = kFp4 ? p.K / 2 : p.K;
+  const int64_t k_bytes = kFp4 ? p.K / 2 : kBf16 ? p.K * 2 : p.K;
   const int num_kb = (int)((k_bytes + kRowBytes - 1) / kRowBytes);
   const int k_steps = (int)(k_bytes / 32);
 
@@ -298,7 +300,9 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
     // ------------------------------------------------------- MMA issuer ---
     if (lane == 0 && leader) {
       constexpr int kMmaM = kPair ? 256 : 128;
-      const uint32_t idesc = kFp4 ? idesc_nvfp4(kBN, kMmaM) : idesc_fp8(kBN, kMmaM);
+      const uint32_t idesc = kFp4    ? idesc_nvfp4(kBN, kMmaM)
+                             : kBf16 ? idesc_bf16(kBN, kMmaM)
+                                     : idesc_fp8(kBN, kMmaM);
       // A stage is ready for its MMAs once its operands have landed (full)
       // and, for NVFP4, its scales are in TMEM (sf_ready).
       auto wait_ready = [&](int st, uint32_t ph) {
@@ -328,6 +332,11 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
                 mma_nvfp4_pair(d_tmem, adesc, bdesc, idesc, sfa_t, sfa_t + 4, accumulate);
               else
                 mma_nvfp4(d_tmem, adesc, bdesc, idesc, sfa_t, sfa_t + 4, accumulate);
+            } else if (kBf16) {
+              if (kPair)
+                mma_bf16_pair(d_tmem, adesc, bdesc, idesc, accumulate);
+              else
+                mma_bf16(d_tmem, adesc, bdesc, idesc, accumulate);
             } else {
               if (kPair)
                 mma_fp8_pair(d_tmem, adesc, bdesc, idesc, accumulate);
@@ -454,8 +463,8 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
     const int quarter = warp & 3;   // the TMEM lane quarter this warp may access
     const int half = e >> 2;
     uint8_t* const out_buf = out_stage + e * 4096;   // this warp's two staging boxes
-    const float sdec_a = *p.sdec_a;
-    const float alpha = kFp4 ? __fmul_rn(sdec_a, *p.sdec_w) : 0.0f;
+    const float sdec_a = kBf16 ? 1.0f : *p.sdec_a;
+    const float alpha = kFp4 ? __fmul_rn(sdec_a, *p.sdec_w) : kBf16 ? 1.0f : 0.0f;
     float s_enc_next = 0.0f;
     if (kRequant) {
       const float s_next = *p.next_scale;
@@ -507,7 +516,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
         for (int b = 0; b < kBatch; ++b) {
           const int c = cb + b;
           float a[32];
-          if (kFp4) {
+          if (kFp4 || kBf16) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) a[i] = alpha;
           } else {
@@ -681,12 +690,14 @@ CUresult encode_4d(CUtensorMap* map, CUtensorMapDataType type, const void* base,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
-// Codes [rows, k_bytes] as a 4-D tensor with two unit dimensions, 128-byte x
-// box_rows boxes with the 128-byte swizzle.
+// Codes [rows, k_bytes] (row stride row_stride bytes, 0 = packed) as a 4-D
+// tensor with two unit dimensions, 128-byte x box_rows boxes with the
+// 128-byte swizzle.
 CUresult encode_codes(CUtensorMap* map, const void* base, uint64_t k_bytes, uint64_t rows,
-                      uint32_t box_rows) {
+                      uint32_t box_rows, uint64_t row_stride = 0) {
+  const uint64_t st = row_stride ? row_stride : k_bytes;
   const cuuint64_t dims[4] = {k_bytes, rows, 1, 1};
-  const cuuint64_t strides[3] = {k_bytes, k_bytes * rows, k_bytes * rows};
+  const cuuint64_t strides[3] = {st, st * rows, st * rows};
   const cuuint32_t box[4] = {kRowBytes, box_rows, 1, 1};
   return encode_4d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base, dims, strides, box,
                    CU_TENSOR_MAP_SWIZZLE_128B);
@@ -707,17 +718,18 @@ CUresult encode_scales(CUtensorMap* map, const void* base, uint64_t rows, uint64
                    CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
-template <bool kFp4, int kBN, bool kPair, bool kRequant>
+template <bool kFp4, int kBN, bool kPair, bool kRequant, bool kBf16 = false>
 cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned* err,
                        uint64_t timeout_ns) {
   using C = Cfg<kFp4, kBN, kPair>;
   constexpr int kCM = kPair ? 2 : 1;
-  const uint64_t k_bytes = kFp4 ? (uint64_t)a.K / 2 : (uint64_t)a.K;
+  const uint64_t k_bytes = kFp4 ? (uint64_t)a.K / 2 : kBf16 ? (uint64_t)a.K * 2 : (uint64_t)a.K;
   CUtensorMap ta, tb, tsa, tsb, ty;
   std::memset(&tsa, 0, sizeof tsa);
   std::memset(&tsb, 0, sizeof tsb);
   std::memset(&ty, 0, sizeof ty);
-  if (encode_codes(&ta, a.a_codes, k_bytes, (uint64_t)a.M, kBM / kSplit) != CUDA_SUCCESS ||
+  if (encode_codes(&ta, a.a_codes, k_bytes, (uint64_t)a.M, kBM / kSplit,
+                   (uint64_t)a.a_row_bytes) != CUDA_SUCCESS ||
       encode_codes(&tb, a.w_codes, k_bytes, (uint64_t)a.N, kBN / kCM / kSplit) != CUDA_SUCCESS ||
       (kFp4 && (encode_scales(&tsa, a.sfa, (uint64_t)a.M, (uint64_t)a.K, 1) != CUDA_SUCCESS ||
                 encode_scales(&tsb, a.sfb, (uint64_t)a.N, (uint64_t)a.K, C::kSfbAtoms) !=
@@ -744,7 +756,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   p.y_amax = a.y_amax;
   p.err = err;
   p.timeout_ns = timeout_ns;
-  auto kern = gemm_kernel<kFp4, kBN, kPair, kRequant>;
+  auto kern = gemm_kernel<kFp4, kBN, kPair, kRequant, kBf16>;
 
   cudaLaunchConfig_t cfg{};
   cudaLaunchAttribute attr[2];
@@ -829,6 +841,12 @@ CUresult encode_tensor_map_out_bf16(CUtensorMap* map, void* base, uint64_t cols,
 
 cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned* err,
                         uint64_t timeout_ns) {
+  if (a.bf16) {
+    const int64_t tiles256 = ((a.M + kBM - 1) / kBM) * ((a.N + 255) / 256);
+    return tiles256 >= num_sms
+               ? launch_cfg<false, 256, true, false, true>(a, s, num_sms, err, timeout_ns)
+               : launch_cfg<false, 128, false, false, true>(a, s, num_sms, err, timeout_ns);
+  }
   return a.fp4 ? dispatch_bn<true>(a, s, num_sms, err, timeout_ns)
                : dispatch_bn<false>(a, s, num_sms, err, timeout_ns);
 }

@@ -40,7 +40,9 @@ cudaError_t launch_quant_fp8_rows(const void* w, int64_t N, int64_t K, const qli
 // ---- GEMMs (qlin_gemm.cu) ----
 struct GemmArgs {
   bool fp4;                 // NVFP4 (true) or FP8
-  const void* a_codes;      // [M, K/2] or [M, K] bytes
+  bool bf16;                // bf16 operands (fp4 false), no scales
+  const void* a_codes;      // [M, K/2] or [M, K] bytes, or bf16 [M, K]
+  int64_t a_row_bytes;      // row stride of A in bytes (0: packed rows)
   const void* w_codes;      // [N, K/2] or [N, K] bytes
   const uint8_t* sfa;       // swizzled block scales (NVFP4)
   const uint8_t* sfb;

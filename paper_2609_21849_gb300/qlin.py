@@ -24,7 +24,7 @@ STATUS = {0: "QLIN_OK", 1: "QLIN_ERR_INVALID_ARG", 2: "QLIN_ERR_UNSUPPORTED",
 # Every function declared in include/qlin.h.
 EXPORTS = ("qlin_nvfp4_scale_bytes", "qlin_workspace_size", "qlin_quantize_act_nvfp4",
            "qlin_quantize_act_fp8", "qlin_quantize_weight", "qlin_gemm_nvfp4", "qlin_gemm_fp8",
-           "qlin_linear_fused", "qlin_linear_dynamic", "qlin_quantize_act_nvfp4_noalloc",
+           "qlin_linear_fused", "qlin_linear_dynamic", "qlin_gemm_bf16", "qlin_quantize_act_nvfp4_noalloc",
            "qlin_sync_status", "qlin_selftest_bounded_wait",
            "qlin_set_wait_timeout_ns", "qlin_status_str", "qlin_last_error")
 
@@ -72,6 +72,7 @@ def load_library(path: str = LIB_PATH):
             "qlin_gemm_fp8": (ctypes.c_int, [ctypes.POINTER(FP8Desc), ctypes.POINTER(FP8Desc), p, p]),
             "qlin_linear_fused": (ctypes.c_int, [ctypes.POINTER(NVFP4Desc), ctypes.POINTER(NVFP4Desc), p, p,
                                                  ctypes.POINTER(NVFP4Desc), i64, p]),
+            "qlin_gemm_bf16": (ctypes.c_int, [p, i64, p, i64, i64, i64, p, p]),
             "qlin_linear_dynamic": (ctypes.c_int, [ctypes.POINTER(NVFP4Desc), ctypes.POINTER(NVFP4Desc), p,
                                                    ctypes.POINTER(NVFP4Desc), p, sz, p]),
             "qlin_quantize_act_nvfp4_noalloc": (ctypes.c_int, [p, i64, i64, ctypes.POINTER(NVFP4Desc), p]),
@@ -274,6 +275,21 @@ def qlin_linear_fused(A: NVFP4Tensor, W: NVFP4Tensor, y: torch.Tensor | None,
         ctypes.byref(dq) if dq is not None else None, rq_col0, _stream(stream)),
         "qlin_linear_fused")
     return y, y_q
+
+
+def qlin_gemm_bf16(a: torch.Tensor, w: torch.Tensor, y: torch.Tensor | None = None, stream=None):
+    """y = a w^T for bf16 a [M, K] (rows may be strided: any view with unit
+    column stride) and w [N, K]; bf16 y [M, N]."""
+    if a.dtype != torch.bfloat16 or w.dtype != torch.bfloat16 or a.dim() != 2 or a.stride(1) != 1:
+        raise ValueError("a, w: bf16 matrices with unit column stride")
+    w = w.contiguous()
+    M, K = a.shape
+    N = w.shape[0]
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.bfloat16, device=a.device)
+    _check(load_library().qlin_gemm_bf16(_ptr(a), a.stride(0), _ptr(w), M, N, K, _ptr(y),
+                                         _stream(stream)), "qlin_gemm_bf16")
+    return y
 
 
 def qlin_linear_dynamic(A: NVFP4Tensor, W: NVFP4Tensor, y: torch.Tensor | None = None,

@@ -80,6 +80,10 @@ def test_argument_errors_return_before_launch(lib):
                                    None) == 6
     assert lib.qlin_linear_dynamic(ctypes.byref(a), ctypes.byref(w), None, ctypes.byref(q), 16, 256,
                                    None) == 1
+    # bf16 GEMM: K not a multiple of 64, row stride below K, misaligned row stride
+    assert lib.qlin_gemm_bf16(16, 96, 16, 128, 128, 96, 16, None) == 1
+    assert lib.qlin_gemm_bf16(16, 64, 16, 128, 128, 128, 16, None) == 1
+    assert lib.qlin_gemm_bf16(16, 132, 16, 128, 128, 128, 16, None) == 3
     # FP8: per-channel activation descriptor is rejected; unknown weight format
     f = qlin.FP8Desc(16, 16, 128, 256, 1)
     assert lib.qlin_quantize_act_fp8(16, 128, 256, 16, ctypes.byref(f), None, 0, None) == 1
