@@ -480,6 +480,57 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
         del st, x, g
         torch.cuda.empty_cache()
     rows["a9_stack"] = res
+
+    # precision ladder (Table 2's BF16 / FP8 / NVFP4 axis) on the same 8-block
+    # stack at B = 1, every linear chained from the bf16 stack input:
+    #  bf16:  unquantized linears (QKV's value columns feed the out-projection
+    #         as a strided view);
+    #  fp8:   W8A8, per-channel weight scales, static calibrated activation
+    #         scales, each epilogue writing the next layer's FP8 input;
+    #  nvfp4: the fused NVFP4 chain (the a9 B = 1 forward).
+    x = to_dev(synthetic.stack_input(1), torch)
+    M1 = x.shape[0]
+    V0 = 2 * synthetic.HIDDEN
+    wbf = [(name, to_dev(wb_, torch)) for (_, name, wb_) in wlist]
+    ybf = [torch.empty((M1, w.shape[0]), dtype=torch.bfloat16, device="cuda") for _, w in wbf]
+
+    def fwd_bf16():
+        a = x
+        for (name, w), y in zip(wbf, ybf):
+            qlin.qlin_gemm_bf16(a, w, y)
+            a = y[:, V0:] if name == "qkv" else y
+    w8 = [(name, qlin.qlin_quantize_weight(w, qlin.QLIN_FMT_FP8)) for name, w in wbf]
+    win = [(V0, w.shape[0] - V0) if name == "qkv" else (0, w.shape[0]) for name, w in wbf]
+    a8 = [qlin.qlin_quantize_act_fp8(x)] + [qlin.alloc_fp8(M1, n, False) for (_, n) in win]
+    nxt8 = [torch.ones(1, dtype=torch.float32, device="cuda") for _ in w8]
+    for i, ((name, W), (c0, n)) in enumerate(zip(w8, win)):   # calibration
+        qlin.qlin_gemm_fp8(a8[i], W, ybf[i])
+        qlin.qlin_quantize_act_fp8(ybf[i][:, c0:c0 + n].contiguous(), None, a8[i + 1])
+        nxt8[i].copy_(a8[i + 1].scale)
+
+    def fwd_fp8():
+        qlin.qlin_quantize_act_fp8(x, None, a8[0], wsp[0])
+        for i, ((name, W), (c0, n)) in enumerate(zip(w8, win)):
+            qlin.qlin_linear_fused_fp8(a8[i], W, ybf[i], nxt8[i], a8[i + 1], c0)
+    st = stack.build_stack(1, weights=wlist)
+    st.calibrate(x)
+
+    def fwd_nvfp4():
+        st.forward(x)
+    ladder = {}
+    for tag, fn in (("bf16", fwd_bf16), ("fp8", fwd_fp8), ("nvfp4", fwd_nvfp4)):
+        fn()
+        torch.cuda.synchronize()
+        g = graph_of(fn, torch, stream)
+        g.replay()
+        t = timed(g.replay, 5, torch, stream)
+        ladder[tag] = {"ms": round(t * 1e3, 3), "TFLOP/s": round(st.flops / t / 1e12, 1)}
+        del g
+    for tag in ("fp8", "nvfp4"):
+        ladder[tag]["speedup_vs_bf16"] = round(ladder["bf16"]["ms"] / ladder[tag]["ms"], 2)
+    rows["f2_precision_ladder_stack_B1"] = ladder
+    del wbf, ybf, w8, a8, st
+    torch.cuda.empty_cache()
     return rows
 
 

@@ -227,6 +227,23 @@ qlin_status qlin_quantize_act_nvfp4_noalloc(const void *x_bf16, int64_t M, int64
                                             qlin_nvfp4_t *out, void *stream);
 
 /*
+ * FP8 linear with the next layer's FP8 input written by the epilogue (Sec. 4:
+ * W8A8 layers in a chain, post-training static activation scale): as
+ * qlin_gemm_fp8, and columns [rq_col0, rq_col0 + y_q->K) of bf16(y) are
+ * quantized to E4M3 with the static S_dec *next_scale:
+ *   code = E4M3_rn_sat(bf16(y) * S_enc), S_enc = 1 / S_dec (FLT_MAX if that
+ *   overflows) -- the FP8 activation quantizer's arithmetic.
+ *  y_bf16:     may be NULL (only the quantized output is written).
+ *  next_scale: device fp32 S_dec, required.
+ *  y_q:        per-tensor FP8 operand, rows == A->rows, K % 64 == 0; its
+ *              scale receives S_dec.  rq_col0 % 64 == 0.
+ * Errors: INVALID_ARG, MISALIGNED, UNSUPPORTED, CUDA.
+ */
+qlin_status qlin_linear_fused_fp8(const qlin_fp8_t *A, const qlin_fp8_t *W, void *y_bf16,
+                                  const float *next_scale, qlin_fp8_t *y_q, int64_t rq_col0,
+                                  void *stream);
+
+/*
  * Unquantized bf16 linear on the same tensor-core skeleton (tcgen05
  * kind::f16), the reference precision of Table 2 (BF16 / FP8 / NVFP4 step
  * latencies): y = a w^T, fp32 accumulation, bf16 out.

@@ -250,7 +250,8 @@ qlin_status qlin_quantize_weight(const void* w_bf16, int64_t N, int64_t K, qlin_
 
 static qlin_status gemm_common(bool fp4, const void* Aany, const void* Wany, void* y,
                                const float* next_scale, qlin_nvfp4_t* y_q, int64_t rq_col0,
-                               void* stream, unsigned* y_amax = nullptr) {
+                               void* stream, unsigned* y_amax = nullptr,
+                               qlin_fp8_t* y_q8 = nullptr) {
   GemmArgs a{};
   a.y_amax = y_amax;
   a.fp4 = fp4;
@@ -290,17 +291,27 @@ static qlin_status gemm_common(bool fp4, const void* Aany, const void* Wany, voi
   if (y != nullptr && !aligned(y, 16)) return QLIN_ERR_MISALIGNED;
   a.y = y;
   if (next_scale != nullptr) {
-    if (y_q == nullptr || !aligned(next_scale, 4)) return QLIN_ERR_INVALID_ARG;
-    if (y_q->K < 64 || y_q->K % 64 != 0 || rq_col0 < 0 || rq_col0 % 64 != 0 ||
-        rq_col0 + y_q->K > a.N)
+    // the re-quantized operand: NVFP4 after an NVFP4 GEMM, FP8 after an FP8 one
+    const int64_t rq_cols = fp4 ? (y_q ? y_q->K : 0) : (y_q8 ? y_q8->K : 0);
+    if ((fp4 ? y_q == nullptr : y_q8 == nullptr) || !aligned(next_scale, 4))
       return QLIN_ERR_INVALID_ARG;
-    QLIN_TRY(check_nvfp4(y_q, a.M, y_q->K));
+    if (rq_cols < 64 || rq_cols % 64 != 0 || rq_col0 < 0 || rq_col0 % 64 != 0 ||
+        rq_col0 + rq_cols > a.N)
+      return QLIN_ERR_INVALID_ARG;
+    if (fp4) {
+      QLIN_TRY(check_nvfp4(y_q, a.M, y_q->K));
+      a.rq_codes = y_q->codes;
+      a.rq_scales = y_q->scales;
+      a.rq_tensor_scale = y_q->tensor_scale;
+    } else {
+      QLIN_TRY(check_fp8(y_q8, a.M, y_q8->K));
+      if (y_q8->per_channel) return QLIN_ERR_INVALID_ARG;
+      a.rq_codes = y_q8->codes;
+      a.rq_tensor_scale = y_q8->scale;
+    }
     a.next_scale = next_scale;
-    a.rq_codes = y_q->codes;
-    a.rq_scales = y_q->scales;
-    a.rq_tensor_scale = y_q->tensor_scale;
     a.rq_col0 = rq_col0;
-    a.rq_cols = y_q->K;
+    a.rq_cols = rq_cols;
   } else if (y == nullptr) {
     return QLIN_ERR_INVALID_ARG;  // nothing to write
   }
@@ -375,6 +386,13 @@ qlin_status qlin_linear_dynamic(const qlin_nvfp4_t* A, const qlin_nvfp4_t* W, vo
   QLIN_CUDA(launch_quant_nvfp4(y_bf16, A->rows, W->rows, reinterpret_cast<const float*>(amax),
                                true, *y_q, s, sms, status, timeout()));
   return QLIN_OK;
+}
+
+qlin_status qlin_linear_fused_fp8(const qlin_fp8_t* A, const qlin_fp8_t* W, void* y_bf16,
+                                  const float* next_scale, qlin_fp8_t* y_q, int64_t rq_col0,
+                                  void* stream) {
+  if (next_scale == nullptr) return QLIN_ERR_INVALID_ARG;
+  return gemm_common(false, A, W, y_bf16, next_scale, nullptr, rq_col0, stream, nullptr, y_q);
 }
 
 qlin_status qlin_sync_status(void* stream) {

@@ -580,7 +580,29 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
         }
       }
       if (row < p.M) {
-        if (kRequant) {
+        if (kRequant && !kFp4) {
+          // FP8 re-quantization with the static next-layer scale: E4M3 of
+          // bf16(y) * S_enc per element, 64 columns per group
+#pragma unroll
+          for (int g = 0; g < kCols / 64; ++g) {
+            const int64_t c64 = col0 + g * 64;
+            if (c64 < p.rq_col0 || c64 + 64 > p.rq_col0 + p.rq_cols || c64 >= p.N) continue;
+            uint8_t* cp = p.rq_codes + row * p.rq_cols + (c64 - p.rq_col0);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {   // 16 columns per 16-byte store
+              const uint32_t* pk = packed + g * 32 + q * 8;
+              uint32_t w4[4];
+#pragma unroll
+              for (int i = 0; i < 4; ++i)
+                w4[i] = e4m3x4(__fmul_rn(bf16_lo(pk[2 * i]), s_enc_next),
+                               __fmul_rn(bf16_hi(pk[2 * i]), s_enc_next),
+                               __fmul_rn(bf16_lo(pk[2 * i + 1]), s_enc_next),
+                               __fmul_rn(bf16_hi(pk[2 * i + 1]), s_enc_next));
+              st_global_v4(cp + 16 * q, w4[0], w4[1], w4[2], w4[3]);
+            }
+          }
+        }
+        if (kRequant && kFp4) {
 #pragma unroll
           for (int g = 0; g < kCols / 64; ++g) {
             const int64_t c64 = col0 + g * 64;
@@ -801,11 +823,9 @@ cudaError_t dispatch_bn(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned
   // single-CTA tiles (small M).
   const int64_t tiles256 = ((a.M + kBM - 1) / kBM) * ((a.N + 255) / 256);
   const bool wide = tiles256 >= num_sms;
-  if constexpr (kFp4) {
-    if (a.next_scale != nullptr)
-      return wide ? launch_cfg<true, 256, true, true>(a, s, num_sms, err, timeout_ns)
-                  : launch_cfg<true, 128, false, true>(a, s, num_sms, err, timeout_ns);
-  }
+  if (a.next_scale != nullptr)
+    return wide ? launch_cfg<kFp4, 256, true, true>(a, s, num_sms, err, timeout_ns)
+                : launch_cfg<kFp4, 128, false, true>(a, s, num_sms, err, timeout_ns);
   return wide ? launch_cfg<kFp4, 256, true, false>(a, s, num_sms, err, timeout_ns)
               : launch_cfg<kFp4, 128, false, false>(a, s, num_sms, err, timeout_ns);
 }

@@ -24,7 +24,8 @@ STATUS = {0: "QLIN_OK", 1: "QLIN_ERR_INVALID_ARG", 2: "QLIN_ERR_UNSUPPORTED",
 # Every function declared in include/qlin.h.
 EXPORTS = ("qlin_nvfp4_scale_bytes", "qlin_workspace_size", "qlin_quantize_act_nvfp4",
            "qlin_quantize_act_fp8", "qlin_quantize_weight", "qlin_gemm_nvfp4", "qlin_gemm_fp8",
-           "qlin_linear_fused", "qlin_linear_dynamic", "qlin_gemm_bf16", "qlin_quantize_act_nvfp4_noalloc",
+           "qlin_linear_fused", "qlin_linear_fused_fp8", "qlin_linear_dynamic", "qlin_gemm_bf16",
+           "qlin_quantize_act_nvfp4_noalloc",
            "qlin_sync_status", "qlin_selftest_bounded_wait",
            "qlin_set_wait_timeout_ns", "qlin_status_str", "qlin_last_error")
 
@@ -73,6 +74,8 @@ def load_library(path: str = LIB_PATH):
             "qlin_linear_fused": (ctypes.c_int, [ctypes.POINTER(NVFP4Desc), ctypes.POINTER(NVFP4Desc), p, p,
                                                  ctypes.POINTER(NVFP4Desc), i64, p]),
             "qlin_gemm_bf16": (ctypes.c_int, [p, i64, p, i64, i64, i64, p, p]),
+            "qlin_linear_fused_fp8": (ctypes.c_int, [ctypes.POINTER(FP8Desc), ctypes.POINTER(FP8Desc), p, p,
+                                                     ctypes.POINTER(FP8Desc), i64, p]),
             "qlin_linear_dynamic": (ctypes.c_int, [ctypes.POINTER(NVFP4Desc), ctypes.POINTER(NVFP4Desc), p,
                                                    ctypes.POINTER(NVFP4Desc), p, sz, p]),
             "qlin_quantize_act_nvfp4_noalloc": (ctypes.c_int, [p, i64, i64, ctypes.POINTER(NVFP4Desc), p]),
@@ -274,6 +277,17 @@ def qlin_linear_fused(A: NVFP4Tensor, W: NVFP4Tensor, y: torch.Tensor | None,
         ctypes.byref(da), ctypes.byref(dw), _ptr(y), _ptr(next_scale),
         ctypes.byref(dq) if dq is not None else None, rq_col0, _stream(stream)),
         "qlin_linear_fused")
+    return y, y_q
+
+
+def qlin_linear_fused_fp8(A: FP8Tensor, W: FP8Tensor, y: torch.Tensor | None,
+                          next_scale: torch.Tensor, y_q: FP8Tensor, rq_col0: int = 0, stream=None):
+    """FP8 linear whose epilogue also writes the next layer's FP8 input
+    (columns [rq_col0, rq_col0 + y_q.K) of bf16(y), static scale)."""
+    da, dw, dq = A.desc(), W.desc(), y_q.desc()
+    _check(load_library().qlin_linear_fused_fp8(
+        ctypes.byref(da), ctypes.byref(dw), _ptr(y), _ptr(next_scale), ctypes.byref(dq), rq_col0,
+        _stream(stream)), "qlin_linear_fused_fp8")
     return y, y_q
 
 

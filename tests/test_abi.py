@@ -80,6 +80,12 @@ def test_argument_errors_return_before_launch(lib):
                                    None) == 6
     assert lib.qlin_linear_dynamic(ctypes.byref(a), ctypes.byref(w), None, ctypes.byref(q), 16, 256,
                                    None) == 1
+    # FP8 fused re-quantization without its static scale
+    f8 = qlin.FP8Desc(16, 16, 128, 256, 0)
+    f8w = qlin.FP8Desc(16, 16, 256, 256, 1)
+    f8q = qlin.FP8Desc(16, 16, 128, 256, 0)
+    assert lib.qlin_linear_fused_fp8(ctypes.byref(f8), ctypes.byref(f8w), 16, None, ctypes.byref(f8q),
+                                     0, None) == 1
     # bf16 GEMM: K not a multiple of 64, row stride below K, misaligned row stride
     assert lib.qlin_gemm_bf16(16, 96, 16, 128, 128, 96, 16, None) == 1
     assert lib.qlin_gemm_bf16(16, 64, 16, 128, 128, 128, 16, None) == 1
