@@ -531,6 +531,62 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
     rows["f2_precision_ladder_stack_B1"] = ladder
     del wbf, ybf, w8, a8, st
     torch.cuda.empty_cache()
+
+    # weight streaming (Sec. 4, "Weight streaming") on the NVFP4 stack: a
+    # resident fraction of the layers, the rest copied from pinned host memory
+    # through two device slots.  M is the measured pinned host -> device rate;
+    # L the resident forward's time per linear; W a streamed layer's bytes.
+    # "model_ms" is the event-level timing of the two-slot schedule with
+    # per-layer L split by FLOPs; "delta_ms" the paper's (N - K) * W / M with
+    # N - K the layers that model finds waiting on their copy.
+    from paper_2609_21849_gb300 import streaming
+    big = max(wlist, key=lambda t: t[2].size)[2].shape
+    hb = torch.empty(big[0] * big[1] // 2 + qlin.qlin_nvfp4_scale_bytes(*big), dtype=torch.uint8).pin_memory()
+    db = torch.empty_like(hb, device="cuda")
+    db.copy_(hb, non_blocking=True)
+    t_cp = timed(lambda: db.copy_(hb, non_blocking=True), 20, torch, torch.cuda.current_stream())
+    M_rate = hb.numel() / t_cp
+    del hb, db
+    stream_rows = {"M_GB/s": round(M_rate / 1e9, 1)}
+    for B in (1, 4):
+        st = stack.build_stack(B, weights=wlist)
+        x = to_dev(synthetic.stack_input(B), torch)
+        st.calibrate(x)
+        st.forward(x)
+        torch.cuda.synchronize()
+        g = graph_of(lambda: st.forward(x), torch, stream)
+        g.replay()
+        t_res = timed(g.replay, 5, torch, stream)
+        del g
+        n = len(st.layers)
+        wbytes = [l.W.codes.numel() + l.W.scales.numel() for l in st.layers]
+        fl = [2 * st.M * l.N * l.K for l in st.layers]
+        L_i = [t_res * f / st.flops for f in fl]
+        C_i = [w / M_rate for w in wbytes]
+        W_mean = sum(wbytes) / n
+        res = {"resident_ms": round(t_res * 1e3, 3),
+               "lambda": round(streaming.reservoir_lambda(t_res / n, M_rate, W_mean), 3)}
+        for frac in (0.75, 0.5, 0.25, 0.0):
+            ss = streaming.StreamedStack(st, frac, release=False)
+            ss.forward(x, stream)
+            torch.cuda.synchronize()
+            g = graph_of(lambda: ss.forward(x, stream), torch, stream)
+            g.replay()
+            t = timed(g.replay, 5, torch, stream)
+            model_t, awaited = streaming.simulate(ss.resident, L_i, C_i)
+            dev_w = sum(w for w, r in zip(wbytes, ss.resident) if r) + ss.slot_bytes
+            res[f"ws{int(frac * 100)}"] = {
+                "ms": round(t * 1e3, 3), "overhead_pct": round((t / t_res - 1) * 100, 1),
+                "model_ms": round(model_t * 1e3, 3), "awaited_layers": awaited,
+                "delta_ms": round(streaming.predicted_overhead(n, n - awaited, W_mean, M_rate) * 1e3, 3),
+                "device_weight_MB": round(dev_w / 1e6, 1)}
+            del g, ss
+        res["all_resident_weight_MB"] = round(sum(wbytes) / 1e6, 1)
+        assert qlin.qlin_sync_status() == 0
+        stream_rows[f"B{B}"] = res
+        del st, x
+        torch.cuda.empty_cache()
+    rows["f3_weight_streaming_stack"] = stream_rows
     return rows
 
 

@@ -1,0 +1,103 @@
+"""Host logic of weight streaming (Sec. 4, "Weight streaming"): which layers
+stay resident, the two-slot copy plan, and the timing model of that schedule
+against the paper's closed forms (lambda = L*M/W; Delta = (N-K)*W/M when the
+reservoir drains; T_min = 2*W_max + A_max)."""
+import itertools
+import math
+
+import pytest
+
+from paper_2609_21849_gb300 import streaming as ws
+
+
+@pytest.mark.parametrize("n", [1, 4, 7, 32])
+def test_resident_layers_count_and_spread(n):
+    for frac in [0.0, 0.1, 0.25, 0.4, 0.5, 0.75, 1.0]:
+        r = ws.resident_layers(n, frac)
+        k = round(frac * n)
+        assert len(r) == n and sum(r) == k
+        if k:
+            assert r[0]                                   # first layer never waits on a copy
+            idx = [i for i, v in enumerate(r) if v]
+            gaps = [b - a for a, b in zip(idx, idx[1:] + [idx[0] + n])]
+            assert max(gaps) - min(gaps) <= 1             # evenly spread
+
+
+def test_copy_plan_alternates_slots():
+    r = [True, False, False, True, False, False, False]
+    assert ws.copy_plan(r) == [(1, 0), (2, 1), (4, 0), (5, 1), (6, 0)]
+    assert ws.copy_plan([True] * 5) == []
+    assert [s for _, s in ws.copy_plan([False] * 6)] == [0, 1, 0, 1, 0, 1]
+
+
+def test_compute_bound_reservoir_adds_nothing():
+    # lambda >= 1 on every layer and the first layer resident: no added latency
+    for n, frac in itertools.product([4, 16, 32], [0.25, 0.5, 0.75]):
+        r = ws.resident_layers(n, frac)
+        L, W, M = 2.0e-4, 2.0e7, 1.0e11                   # lambda = L*M/W = 1
+        assert ws.reservoir_lambda(L, M, W) == pytest.approx(1.0)
+        t, awaited = ws.simulate(r, L, W / M)
+        assert t == pytest.approx(n * L) and awaited == 0
+    # everything streamed: only the first copy is exposed
+    t, awaited = ws.simulate([False] * 8, 1.0, 0.5)
+    assert t == pytest.approx(8.5) and awaited == 1
+
+
+def test_copy_bound_limit_equals_closed_form():
+    # with no compute to hide behind, every streamed layer waits its full
+    # transfer: the added latency is exactly (N - K) * W / M
+    n, W, M = 32, 2.1e7, 3.0e11
+    for frac in [0.0, 0.25, 0.5, 0.75, 1.0]:
+        r = ws.resident_layers(n, frac)
+        k = sum(r)
+        t, awaited = ws.simulate(r, 0.0, W / M)
+        assert awaited == n - k
+        assert t == pytest.approx(ws.predicted_overhead(n, k, W, M))
+
+
+def test_draining_reservoir_between_the_bounds():
+    # lambda < 1: the added latency lies between zero and the closed form with
+    # the awaited layers as N - K, and grows as residency falls
+    n, L, C = 32, 1.0, 3.0
+    prev = -1.0
+    for frac in [1.0, 0.75, 0.5, 0.25, 0.0]:
+        r = ws.resident_layers(n, frac)
+        t, awaited = ws.simulate(r, L, C)
+        extra = t - n * L
+        assert 0.0 <= extra <= awaited * C + 1e-9
+        assert extra >= prev
+        prev = extra
+    # all streamed: the copy engine is the bottleneck, finish = N*C + L
+    t, awaited = ws.simulate([False] * n, L, C)
+    assert t == pytest.approx(n * C + L) and awaited == n
+
+
+def test_simulate_matches_brute_force_schedule():
+    # independent restatement of the two-slot schedule, as a fixed-point over
+    # start times, on every residency pattern of 6 layers
+    import random
+    rng = random.Random(3)
+    for bits in range(64):
+        r = [bool(bits >> i & 1) for i in range(6)]
+        L = [rng.uniform(0.1, 2.0) for _ in r]
+        C = [rng.uniform(0.1, 3.0) for _ in r]
+        streamed = [i for i in range(6) if not r[i]]
+        end = {}
+        cend = {}
+        t = 0.0
+        for i in range(6):
+            if not r[i]:
+                j = streamed.index(i)
+                prev_copy = cend[streamed[j - 1]] if j else 0.0
+                slot_free = end[streamed[j - 2]] if j >= 2 else 0.0
+                cend[i] = max(prev_copy, slot_free) + C[i]
+                t = max(t, cend[i])
+            t += L[i]
+            end[i] = t
+        got, _ = ws.simulate(r, L, C)
+        assert math.isclose(got, t, rel_tol=1e-12), (r, got, t)
+
+
+def test_t_min():
+    # two slots of the largest layer plus the peak activation
+    assert ws.t_min(21_233_664, 113_246_208) == 2 * 21_233_664 + 113_246_208
