@@ -523,7 +523,7 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
         torch.cuda.synchronize()
         g = graph_of(fn, torch, stream)
         g.replay()
-        t = timed(g.replay, 5, torch, stream)
+        t = statistics.median(timed(g.replay, 3, torch, stream) for _ in range(3))
         ladder[tag] = {"ms": round(t * 1e3, 3), "TFLOP/s": round(st.flops / t / 1e12, 1)}
         del g
     for tag in ("fp8", "nvfp4"):
@@ -536,7 +536,8 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
     # resident fraction of the layers, the rest copied from pinned host memory
     # through two device slots.  M is the measured pinned host -> device rate;
     # L the resident forward's time per linear; W a streamed layer's bytes.
-    # "model_ms" is the event-level timing of the two-slot schedule with
+    # Two device slots (the paper's floor) unless "_slotsN" says otherwise.
+    # "model_ms" is the event-level timing of the slot schedule with
     # per-layer L split by FLOPs; "delta_ms" the paper's (N - K) * W / M with
     # N - K the layers that model finds waiting on their copy.
     from paper_2609_21849_gb300 import streaming
@@ -556,7 +557,7 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
         torch.cuda.synchronize()
         g = graph_of(lambda: st.forward(x), torch, stream)
         g.replay()
-        t_res = timed(g.replay, 5, torch, stream)
+        t_res = statistics.median(timed(g.replay, 3, torch, stream) for _ in range(3))
         del g
         n = len(st.layers)
         wbytes = [l.W.codes.numel() + l.W.scales.numel() for l in st.layers]
@@ -566,16 +567,16 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
         W_mean = sum(wbytes) / n
         res = {"resident_ms": round(t_res * 1e3, 3),
                "lambda": round(streaming.reservoir_lambda(t_res / n, M_rate, W_mean), 3)}
-        for frac in (0.75, 0.5, 0.25, 0.0):
-            ss = streaming.StreamedStack(st, frac, release=False)
+        for frac, slots in ((0.75, 2), (0.5, 2), (0.25, 2), (0.0, 2), (0.25, 3), (0.0, 3)):
+            ss = streaming.StreamedStack(st, frac, release=False, n_slots=slots)
             ss.forward(x, stream)
             torch.cuda.synchronize()
             g = graph_of(lambda: ss.forward(x, stream), torch, stream)
             g.replay()
-            t = timed(g.replay, 5, torch, stream)
-            model_t, awaited = streaming.simulate(ss.resident, L_i, C_i)
+            t = statistics.median(timed(g.replay, 3, torch, stream) for _ in range(3))
+            model_t, awaited = streaming.simulate(ss.resident, L_i, C_i, slots)
             dev_w = sum(w for w, r in zip(wbytes, ss.resident) if r) + ss.slot_bytes
-            res[f"ws{int(frac * 100)}"] = {
+            res[f"ws{int(frac * 100)}" + ("" if slots == 2 else f"_slots{slots}")] = {
                 "ms": round(t * 1e3, 3), "overhead_pct": round((t / t_res - 1) * 100, 1),
                 "model_ms": round(model_t * 1e3, 3), "awaited_layers": awaited,
                 "delta_ms": round(streaming.predicted_overhead(n, n - awaited, W_mean, M_rate) * 1e3, 3),

@@ -1,7 +1,7 @@
 """Weight streaming for the denoise-step linear stack (Sec. 4, "Weight
 streaming"): only a resident subset of the layers' weights stays in device
-memory; the others live in pinned host memory and are copied into one of two
-device slots ahead of use, on a copy stream, overlapped with the compute of
+memory; the others live in pinned host memory and are copied into a small
+ring of device slots (two at the memory floor) ahead of use, on a copy stream, overlapped with the compute of
 the layers in between.  Only where the weights live changes, so the outputs
 are bit-identical to a fully resident run.
 
@@ -39,13 +39,14 @@ def resident_layers(n_layers: int, fraction: float) -> list[bool]:
     return res
 
 
-def copy_plan(resident: list[bool]) -> list[tuple[int, int]]:
+def copy_plan(resident: list[bool], n_slots: int = 2) -> list[tuple[int, int]]:
     """(layer, slot) for each streamed layer in execution order; streamed
-    layers alternate between the two device slots."""
+    layers take the device slots round-robin (two slots: layers i and i+1 of
+    the paper's memory floor)."""
     plan, k = [], 0
     for i, r in enumerate(resident):
         if not r:
-            plan.append((i, k % 2))
+            plan.append((i, k % n_slots))
             k += 1
     return plan
 
@@ -61,9 +62,9 @@ def predicted_overhead(n_layers: int, k_overlapped: int, W_bytes: float,
     return (n_layers - k_overlapped) * W_bytes / M_bytes_per_s
 
 
-def simulate(resident: list[bool], L_s, copy_s) -> tuple[float, int]:
-    """Event-level timing of the two-slot schedule that StreamedStack runs
-    (not the paper's closed form): one copy engine takes the streamed layers'
+def simulate(resident: list[bool], L_s, copy_s, n_slots: int = 2) -> tuple[float, int]:
+    """Event-level timing of the slot schedule that StreamedStack runs (not
+    the paper's closed form): one copy engine takes the streamed layers'
     copies in order; the copy into a slot starts once the layer that last read
     the slot has finished; a streamed layer starts once its copy has landed.
     ``L_s`` / ``copy_s``: per-layer compute and copy times (scalars or lists).
@@ -72,8 +73,8 @@ def simulate(resident: list[bool], L_s, copy_s) -> tuple[float, int]:
     n = len(resident)
     L = L_s if isinstance(L_s, (list, tuple)) else [L_s] * n
     C = copy_s if isinstance(copy_s, (list, tuple)) else [copy_s] * n
-    plan = copy_plan(resident)
-    landed, slot_free = {}, [0.0, 0.0]
+    plan = copy_plan(resident, n_slots)
+    landed, slot_free = {}, [0.0] * n_slots
     engine = 0.0
     t = 0.0
     def issue(j):
@@ -81,7 +82,7 @@ def simulate(resident: list[bool], L_s, copy_s) -> tuple[float, int]:
         layer, slot = plan[j]
         engine = max(engine, slot_free[slot]) + C[layer]
         landed[layer] = engine
-    for j in range(min(2, len(plan))):
+    for j in range(min(n_slots, len(plan))):
         issue(j)
     k = awaited = 0
     for i in range(n):
@@ -91,16 +92,16 @@ def simulate(resident: list[bool], L_s, copy_s) -> tuple[float, int]:
         t += L[i]
         if not resident[i]:
             slot_free[plan[k][1]] = t
-            if k + 2 < len(plan):
-                issue(k + 2)
+            if k + n_slots < len(plan):
+                issue(k + n_slots)
             k += 1
     return t, awaited
 
 
-def t_min(w_max_bytes: int, a_max_bytes: int) -> int:
-    """Device memory floor of streaming: two weight slots plus the peak
-    activation."""
-    return 2 * w_max_bytes + a_max_bytes
+def t_min(w_max_bytes: int, a_max_bytes: int, n_slots: int = 2) -> int:
+    """Device memory floor of streaming: the weight slots (two in the paper)
+    plus the peak activation."""
+    return n_slots * w_max_bytes + a_max_bytes
 
 
 # ------------------------------------------------------------- runtime ---
@@ -114,15 +115,20 @@ class _Host:
 
 class StreamedStack:
     """A LinearStack whose non-resident layers' NVFP4 weights are held in
-    pinned host memory and streamed through two device slots.  With
+    pinned host memory and streamed through ``n_slots`` device slots (two by
+    default, the paper's floor; a third lets each copy start one layer
+    earlier, which pays when the copy engine is the bound).  With
     ``release`` the stack's device copies of those weights are dropped (the
     stack then runs only through this object)."""
 
-    def __init__(self, stack, fraction: float, release: bool = True):
+    def __init__(self, stack, fraction: float, release: bool = True, n_slots: int = 2):
+        if n_slots < 2:
+            raise ValueError("weight streaming needs at least two device slots")
+        self.n_slots = n_slots
         self.stack = stack
         n = len(stack.layers)
         self.resident = resident_layers(n, fraction)
-        self.plan = copy_plan(self.resident)
+        self.plan = copy_plan(self.resident, n_slots)
         self.host: dict[int, _Host] = {}
         self.weights = [l.W for l in stack.layers]     # resident layers keep theirs
         cb = sb = 0
@@ -135,12 +141,13 @@ class StreamedStack:
             cb, sb = max(cb, W.codes.numel()), max(sb, W.scales.numel())
             self.weights[i] = None                       # device copy released
         dev = stack.a0.codes.device
-        self.slot_codes = [torch.empty(cb, dtype=torch.uint8, device=dev) for _ in range(2)]
-        self.slot_scales = [torch.empty(sb, dtype=torch.uint8, device=dev) for _ in range(2)]
-        self.slot_ts = [torch.empty(1, dtype=torch.float32, device=dev) for _ in range(2)]
+        ns = n_slots if self.plan else 0
+        self.slot_codes = [torch.empty(cb, dtype=torch.uint8, device=dev) for _ in range(ns)]
+        self.slot_scales = [torch.empty(sb, dtype=torch.uint8, device=dev) for _ in range(ns)]
+        self.slot_ts = [torch.empty(1, dtype=torch.float32, device=dev) for _ in range(ns)]
         self.copy_stream = torch.cuda.Stream(device=dev)
-        self.copied = [torch.cuda.Event() for _ in range(2)]   # slot filled
-        self.freed = [torch.cuda.Event() for _ in range(2)]    # slot's last reader done
+        self.copied = [torch.cuda.Event() for _ in range(ns)]   # slot filled
+        self.freed = [torch.cuda.Event() for _ in range(ns)]    # slot's last reader done
         if release:
             for l, w in zip(stack.layers, self.weights):
                 if w is None:
@@ -174,8 +181,8 @@ class StreamedStack:
         stream = stream if stream is not None else torch.cuda.current_stream()
         for e in self.freed:
             e.record(stream)
-        # the first two streamed layers' copies start at once
-        for layer, slot in self.plan[:2]:
+        # the first n_slots streamed layers' copies start at once
+        for layer, slot in self.plan[:self.n_slots]:
             self._issue_copy(layer, slot)
         if x is not None:
             st.quantize_input(x, stream)
@@ -192,8 +199,8 @@ class StreamedStack:
                                    l.rq_col0, stream)
             if not self.resident[i]:
                 self.freed[slot].record(stream)
-                if k + 2 < len(self.plan):             # refill this slot two copies ahead
-                    self._issue_copy(*self.plan[k + 2])
+                if k + self.n_slots < len(self.plan):  # refill this slot
+                    self._issue_copy(*self.plan[k + self.n_slots])
                 k += 1
             a = l.out_q
         if self.plan:                                  # join the copy stream back

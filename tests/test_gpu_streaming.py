@@ -34,17 +34,18 @@ def test_streamed_forward_bit_identical(B):
     assert qlin.qlin_sync_status() == 0
     ref = _outputs(st)
 
-    for frac, release in [(0.75, False), (0.5, False), (0.25, False), (0.0, True)]:
+    for frac, slots, release in [(0.75, 2, False), (0.5, 2, False), (0.25, 2, False),
+                                 (0.25, 3, False), (0.0, 3, False), (0.0, 2, True)]:
         for l in st.layers:                        # stale outputs must be overwritten
             l.y.zero_(); l.out_q.codes.zero_(); l.out_q.scales.zero_()
-        ss = streaming.StreamedStack(st, frac, release=release)
+        ss = streaming.StreamedStack(st, frac, release=release, n_slots=slots)
         s = torch.cuda.Stream()
         with torch.cuda.stream(s):
             ss.forward(x, s)
             ss.forward(x, s)                       # slots reused across forwards
         torch.cuda.synchronize()
         assert qlin.qlin_sync_status() == 0
-        _assert_same(st, ref, frac)
+        _assert_same(st, ref, (frac, slots))
     assert all(l.W is None for l in st.layers)     # released: only the slots remain
 
 

@@ -72,8 +72,9 @@ def test_draining_reservoir_between_the_bounds():
     assert t == pytest.approx(n * C + L) and awaited == n
 
 
-def test_simulate_matches_brute_force_schedule():
-    # independent restatement of the two-slot schedule, as a fixed-point over
+@pytest.mark.parametrize("n_slots", [2, 3])
+def test_simulate_matches_brute_force_schedule(n_slots):
+    # independent restatement of the slot schedule, as a recurrence over
     # start times, on every residency pattern of 6 layers
     import random
     rng = random.Random(3)
@@ -89,15 +90,30 @@ def test_simulate_matches_brute_force_schedule():
             if not r[i]:
                 j = streamed.index(i)
                 prev_copy = cend[streamed[j - 1]] if j else 0.0
-                slot_free = end[streamed[j - 2]] if j >= 2 else 0.0
+                slot_free = end[streamed[j - n_slots]] if j >= n_slots else 0.0
                 cend[i] = max(prev_copy, slot_free) + C[i]
                 t = max(t, cend[i])
             t += L[i]
             end[i] = t
-        got, _ = ws.simulate(r, L, C)
+        got, _ = ws.simulate(r, L, C, n_slots)
         assert math.isclose(got, t, rel_tol=1e-12), (r, got, t)
+
+
+def test_more_slots_never_slower_and_reach_copy_bound():
+    n, L, C = 32, 1.0, 3.0
+    for frac in [0.75, 0.5, 0.25, 0.0]:
+        r = ws.resident_layers(n, frac)
+        times = [ws.simulate(r, L, C, k)[0] for k in (2, 3, 4, 8)]
+        assert all(b <= a + 1e-9 for a, b in zip(times, times[1:]))
+    # enough slots: the forward runs at max(total compute, total copies)
+    # plus the exposed start
+    r = ws.resident_layers(n, 0.25)
+    t, _ = ws.simulate(r, 0.5, 1.0, n_slots=n)
+    assert t == pytest.approx(24 * 1.0 + 0.5)
 
 
 def test_t_min():
     # two slots of the largest layer plus the peak activation
     assert ws.t_min(21_233_664, 113_246_208) == 2 * 21_233_664 + 113_246_208
+    assert ws.t_min(10, 5, n_slots=3) == 35
+    assert ws.copy_plan([False] * 5, 3) == [(0, 0), (1, 1), (2, 2), (3, 0), (4, 1)]
