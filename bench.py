@@ -481,10 +481,11 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
         torch.cuda.empty_cache()
     rows["a9_stack"] = res
 
-    # precision ladder (Table 2's BF16 / FP8 / NVFP4 axis) on the same 8-block
-    # stack at B = 1, every linear chained from the bf16 stack input:
+    # precision ladder (Table 2's BF16 / FP16 / FP8 / NVFP4 axis) on the same
+    # 8-block stack at B = 1, every linear chained from the stack input:
     #  bf16:  unquantized linears (QKV's value columns feed the out-projection
     #         as a strided view);
+    #  fp16:  the same with fp16 operands;
     #  fp8:   W8A8, per-channel weight scales, static calibrated activation
     #         scales, each epilogue writing the next layer's FP8 input;
     #  nvfp4: the fused NVFP4 chain (the a9 B = 1 forward).
@@ -498,6 +499,19 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
         a = x
         for (name, w), y in zip(wbf, ybf):
             qlin.qlin_gemm_bf16(a, w, y)
+            a = y[:, V0:] if name == "qkv" else y
+    # fp16: the same chain with fp16 operands (converted once, outside the
+    # timed region).  Without the blocks' norms the activations grow about
+    # 3x per block, so the fp16 chain starts from x * 2^-6 (an exact
+    # rescale; its last output would otherwise overflow fp16).
+    x16 = (x.float() * 2.0 ** -6).half()   # exact rescale: keeps the chain inside fp16's range
+    w16 = [(name, w.half()) for name, w in wbf]
+    y16 = [torch.empty_like(y, dtype=torch.float16) for y in ybf]
+
+    def fwd_fp16():
+        a = x16
+        for (name, w), y in zip(w16, y16):
+            qlin.qlin_gemm_fp16(a, w, y)
             a = y[:, V0:] if name == "qkv" else y
     w8 = [(name, qlin.qlin_quantize_weight(w, qlin.QLIN_FMT_FP8)) for name, w in wbf]
     win = [(V0, w.shape[0] - V0) if name == "qkv" else (0, w.shape[0]) for name, w in wbf]
@@ -517,19 +531,36 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
 
     def fwd_nvfp4():
         st.forward(x)
-    ladder = {}
-    for tag, fn in (("bf16", fwd_bf16), ("fp8", fwd_fp8), ("nvfp4", fwd_nvfp4)):
+    # The 16-bit chains run at the power cap (the SM clock drops under
+    # sustained load), so the precisions are timed in interleaved rounds of
+    # about 0.6 s each, with the SM clock sampled during each; "ms_x_ghz"
+    # (time x median clock) compares them per clock cycle.
+    ladder, graphs = {}, {}
+    for tag, fn in (("bf16", fwd_bf16), ("fp16", fwd_fp16), ("fp8", fwd_fp8), ("nvfp4", fwd_nvfp4)):
         fn()
         torch.cuda.synchronize()
-        g = graph_of(fn, torch, stream)
-        g.replay()
-        t = statistics.median(timed(g.replay, 3, torch, stream) for _ in range(3))
-        ladder[tag] = {"ms": round(t * 1e3, 3), "TFLOP/s": round(st.flops / t / 1e12, 1)}
-        del g
-    for tag in ("fp8", "nvfp4"):
+        graphs[tag] = graph_of(fn, torch, stream)
+        graphs[tag].replay()
+    runs = {tag: [] for tag in graphs}
+    for _ in range(3):
+        for tag, g in graphs.items():
+            reps = max(3, int(0.6 / max(timed(g.replay, 1, torch, stream), 1e-4)))
+            clk = Clocks(int(os.environ.get("LOCAL_RANK", 0)))
+            t = timed(g.replay, reps, torch, stream)
+            runs[tag].append((t, clk.stop()))
+    for tag, rs in runs.items():
+        t = statistics.median(r[0] for r in rs)
+        mhz = [r[1]["sm_mhz"] for r in rs if r[1].get("sm_mhz")]
+        reasons = sorted({x for r in rs for x in r[1].get("reasons", [])})
+        ladder[tag] = {"ms": round(t * 1e3, 3), "TFLOP/s": round(st.flops / t / 1e12, 1),
+                       "sm_mhz": statistics.median(mhz) if mhz else None, "reasons": reasons}
+        if mhz:
+            ladder[tag]["ms_x_ghz"] = round(t * 1e3 * statistics.median(mhz) / 1e3, 3)
+    del graphs
+    for tag in ("fp16", "fp8", "nvfp4"):
         ladder[tag]["speedup_vs_bf16"] = round(ladder["bf16"]["ms"] / ladder[tag]["ms"], 2)
     rows["f2_precision_ladder_stack_B1"] = ladder
-    del wbf, ybf, w8, a8, st
+    del wbf, ybf, w8, a8, st, x16, w16, y16
     torch.cuda.empty_cache()
 
     # weight streaming (Sec. 4, "Weight streaming") on the NVFP4 stack: a

@@ -258,6 +258,15 @@ qlin_status qlin_gemm_bf16(const void *a_bf16, int64_t lda, const void *w_bf16, 
                            int64_t N, int64_t K, void *y_bf16, void *stream);
 
 /*
+ * Unquantized fp16 linear: qlin_gemm_bf16 with fp16 operands and an fp16
+ * output, y = fp16_rn(a w^T), fp32 accumulation (Sec. 4: the FP16 engines of
+ * the precision comparison; values beyond 65504 become infinities, as in
+ * any fp16 engine).  Same arguments, layouts and errors as qlin_gemm_bf16.
+ */
+qlin_status qlin_gemm_fp16(const void *a_fp16, int64_t lda, const void *w_fp16, int64_t M,
+                           int64_t N, int64_t K, void *y_fp16, void *stream);
+
+/*
  * Dynamic per-tensor scaling inside a chain of linears (Sec. 4, "Quantization":
  * run-time activation quantization, here with the tensor scale of the layer's
  * own output instead of a calibrated one):

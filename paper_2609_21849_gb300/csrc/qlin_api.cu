@@ -343,20 +343,22 @@ qlin_status qlin_linear_fused(const qlin_nvfp4_t* A, const qlin_nvfp4_t* W, void
   return gemm_common(true, A, W, y_bf16, next_scale, y_q, rq_col0, stream);
 }
 
-qlin_status qlin_gemm_bf16(const void* a_bf16, int64_t lda, const void* w_bf16, int64_t M,
-                           int64_t N, int64_t K, void* y_bf16, void* stream) {
-  if (a_bf16 == nullptr || w_bf16 == nullptr || y_bf16 == nullptr) return QLIN_ERR_INVALID_ARG;
+// The unquantized 16-bit linear (bf16 or fp16 operands and output).
+static qlin_status gemm16(const void* a16, int64_t lda, const void* w16, int64_t M, int64_t N,
+                          int64_t K, void* y16, void* stream, bool fp16) {
+  if (a16 == nullptr || w16 == nullptr || y16 == nullptr) return QLIN_ERR_INVALID_ARG;
   if (M < 1 || K < 64 || K % 64 != 0 || N < 64 || N % 64 != 0 || lda < K)
     return QLIN_ERR_INVALID_ARG;
   if (M > (int64_t)1 << 31 || N > (int64_t)1 << 31) return QLIN_ERR_UNSUPPORTED;
-  if (!aligned(a_bf16, 16) || !aligned(w_bf16, 16) || !aligned(y_bf16, 16) || (lda * 2) % 16 != 0)
+  if (!aligned(a16, 16) || !aligned(w16, 16) || !aligned(y16, 16) || (lda * 2) % 16 != 0)
     return QLIN_ERR_MISALIGNED;
   GemmArgs a{};
   a.bf16 = true;
-  a.a_codes = a_bf16;
+  a.fp16 = fp16;
+  a.a_codes = a16;
   a.a_row_bytes = lda * 2;
-  a.w_codes = w_bf16;
-  a.y = y_bf16;
+  a.w_codes = w16;
+  a.y = y16;
   a.M = M;
   a.N = N;
   a.K = K;
@@ -366,6 +368,16 @@ qlin_status qlin_gemm_bf16(const void* a_bf16, int64_t lda, const void* w_bf16, 
   cudaError_t e = launch_gemm(a, static_cast<cudaStream_t>(stream), sms, status, timeout());
   if (e != cudaSuccess) return cuda_fail(e);
   return QLIN_OK;
+}
+
+qlin_status qlin_gemm_bf16(const void* a_bf16, int64_t lda, const void* w_bf16, int64_t M,
+                           int64_t N, int64_t K, void* y_bf16, void* stream) {
+  return gemm16(a_bf16, lda, w_bf16, M, N, K, y_bf16, stream, false);
+}
+
+qlin_status qlin_gemm_fp16(const void* a_fp16, int64_t lda, const void* w_fp16, int64_t M,
+                           int64_t N, int64_t K, void* y_fp16, void* stream) {
+  return gemm16(a_fp16, lda, w_fp16, M, N, K, y_fp16, stream, true);
 }
 
 qlin_status qlin_linear_dynamic(const qlin_nvfp4_t* A, const qlin_nvfp4_t* W, void* y_bf16,

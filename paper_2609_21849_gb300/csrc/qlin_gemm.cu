@@ -106,6 +106,7 @@ struct KParams {
   float* rq_tensor_scale;
   int64_t rq_col0, rq_cols;
   unsigned* y_amax;   // optional: max |bf16 y| over the output, as fp32 bits (atomicMax)
+  int fp16;           // 16-bit operand kernel only: fp16 operands and output (else bf16)
   unsigned* err;
   uint64_t timeout_ns;
 };
@@ -301,7 +302,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
     if (lane == 0 && leader) {
       constexpr int kMmaM = kPair ? 256 : 128;
       const uint32_t idesc = kFp4    ? idesc_nvfp4(kBN, kMmaM)
-                             : kBf16 ? idesc_bf16(kBN, kMmaM)
+                             : kBf16 ? (p.fp16 ? idesc_fp16(kBN, kMmaM) : idesc_bf16(kBN, kMmaM))
                                      : idesc_fp8(kBN, kMmaM);
       // A stage is ready for its MMAs once its operands have landed (full)
       // and, for NVFP4, its scales are in TMEM (sf_ready).
@@ -537,11 +538,18 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
               for (int i = 0; i < 32; ++i) a[i] = a0;
             }
           }
+          if (kBf16 && p.fp16) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i)
-            packed[c * 16 + i] =
-                pack_bf16x2(__fmul_rn(__uint_as_float(r[b][2 * i]), a[2 * i]),
-                            __fmul_rn(__uint_as_float(r[b][2 * i + 1]), a[2 * i + 1]));
+            for (int i = 0; i < 16; ++i)
+              packed[c * 16 + i] = pack_f16x2(__uint_as_float(r[b][2 * i]),
+                                              __uint_as_float(r[b][2 * i + 1]));
+          } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+              packed[c * 16 + i] =
+                  pack_bf16x2(__fmul_rn(__uint_as_float(r[b][2 * i]), a[2 * i]),
+                              __fmul_rn(__uint_as_float(r[b][2 * i + 1]), a[2 * i + 1]));
+          }
         }
       }
 
@@ -756,8 +764,9 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
       (kFp4 && (encode_scales(&tsa, a.sfa, (uint64_t)a.M, (uint64_t)a.K, 1) != CUDA_SUCCESS ||
                 encode_scales(&tsb, a.sfb, (uint64_t)a.N, (uint64_t)a.K, C::kSfbAtoms) !=
                     CUDA_SUCCESS)) ||
-      (a.y != nullptr && encode_tensor_map_out_bf16(&ty, a.y, (uint64_t)a.N, (uint64_t)a.M) !=
-                             CUDA_SUCCESS))
+      (a.y != nullptr &&
+       encode_tensor_map_out_bf16(&ty, a.y, (uint64_t)a.N, (uint64_t)a.M, kBf16 && a.fp16) !=
+           CUDA_SUCCESS))
     return cudaErrorInvalidValue;
   KParams p{};
   p.sfa = a.sfa;
@@ -776,6 +785,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   p.rq_col0 = a.rq_col0;
   p.rq_cols = a.rq_cols;
   p.y_amax = a.y_amax;
+  p.fp16 = kBf16 && a.fp16 ? 1 : 0;
   p.err = err;
   p.timeout_ns = timeout_ns;
   auto kern = gemm_kernel<kFp4, kBN, kPair, kRequant, kBf16>;
@@ -845,16 +855,18 @@ CUresult encode_tensor_map_2d_u8(CUtensorMap* map, const void* base, uint64_t in
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
-// bf16 [rows, cols] output map: 32 x 32 boxes, 64-byte swizzle (the layout of
-// the epilogue's staging boxes).
-CUresult encode_tensor_map_out_bf16(CUtensorMap* map, void* base, uint64_t cols, uint64_t rows) {
+// bf16 (or fp16) [rows, cols] output map: 32 x 32 boxes, 64-byte swizzle (the
+// layout of the epilogue's staging boxes).
+CUresult encode_tensor_map_out_bf16(CUtensorMap* map, void* base, uint64_t cols, uint64_t rows,
+                                    bool fp16) {
   EncodeTiledFn fn = encode_fn();
   if (fn == nullptr) return CUDA_ERROR_NOT_FOUND;
   const cuuint64_t dims[2] = {cols, rows};
   const cuuint64_t strides[1] = {cols * 2};
   const cuuint32_t box[2] = {32, 32};
   const cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+  return fn(map, fp16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+            base, dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }

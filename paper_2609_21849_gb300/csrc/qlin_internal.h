@@ -40,7 +40,8 @@ cudaError_t launch_quant_fp8_rows(const void* w, int64_t N, int64_t K, const qli
 // ---- GEMMs (qlin_gemm.cu) ----
 struct GemmArgs {
   bool fp4;                 // NVFP4 (true) or FP8
-  bool bf16;                // bf16 operands (fp4 false), no scales
+  bool bf16;                // 16-bit float operands (fp4 false), no scales
+  bool fp16;                // with bf16: the operands and y are fp16, not bf16
   const void* a_codes;      // [M, K/2] or [M, K] bytes, or bf16 [M, K]
   int64_t a_row_bytes;      // row stride of A in bytes (0: packed rows)
   const void* w_codes;      // [N, K/2] or [N, K] bytes
@@ -65,7 +66,8 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned
 cudaError_t launch_wait_selftest(uint64_t timeout_ns, cudaStream_t s, unsigned* err);
 
 // Resolves cuTensorMapEncodeTiled through the runtime (no libcuda link).
-CUresult encode_tensor_map_out_bf16(CUtensorMap* map, void* base, uint64_t cols, uint64_t rows);
+CUresult encode_tensor_map_out_bf16(CUtensorMap* map, void* base, uint64_t cols, uint64_t rows,
+                                    bool fp16 = false);
 CUresult encode_tensor_map_2d_u8(CUtensorMap* map, const void* base, uint64_t inner_bytes,
                                  uint64_t rows, uint32_t box_inner, uint32_t box_rows);
 

@@ -25,7 +25,7 @@ STATUS = {0: "QLIN_OK", 1: "QLIN_ERR_INVALID_ARG", 2: "QLIN_ERR_UNSUPPORTED",
 EXPORTS = ("qlin_nvfp4_scale_bytes", "qlin_workspace_size", "qlin_quantize_act_nvfp4",
            "qlin_quantize_act_fp8", "qlin_quantize_weight", "qlin_gemm_nvfp4", "qlin_gemm_fp8",
            "qlin_linear_fused", "qlin_linear_fused_fp8", "qlin_linear_dynamic", "qlin_gemm_bf16",
-           "qlin_quantize_act_nvfp4_noalloc",
+           "qlin_gemm_fp16", "qlin_quantize_act_nvfp4_noalloc",
            "qlin_sync_status", "qlin_selftest_bounded_wait",
            "qlin_set_wait_timeout_ns", "qlin_status_str", "qlin_last_error")
 
@@ -74,6 +74,7 @@ def load_library(path: str = LIB_PATH):
             "qlin_linear_fused": (ctypes.c_int, [ctypes.POINTER(NVFP4Desc), ctypes.POINTER(NVFP4Desc), p, p,
                                                  ctypes.POINTER(NVFP4Desc), i64, p]),
             "qlin_gemm_bf16": (ctypes.c_int, [p, i64, p, i64, i64, i64, p, p]),
+            "qlin_gemm_fp16": (ctypes.c_int, [p, i64, p, i64, i64, i64, p, p]),
             "qlin_linear_fused_fp8": (ctypes.c_int, [ctypes.POINTER(FP8Desc), ctypes.POINTER(FP8Desc), p, p,
                                                      ctypes.POINTER(FP8Desc), i64, p]),
             "qlin_linear_dynamic": (ctypes.c_int, [ctypes.POINTER(NVFP4Desc), ctypes.POINTER(NVFP4Desc), p,
@@ -291,19 +292,30 @@ def qlin_linear_fused_fp8(A: FP8Tensor, W: FP8Tensor, y: torch.Tensor | None,
     return y, y_q
 
 
-def qlin_gemm_bf16(a: torch.Tensor, w: torch.Tensor, y: torch.Tensor | None = None, stream=None):
-    """y = a w^T for bf16 a [M, K] (rows may be strided: any view with unit
-    column stride) and w [N, K]; bf16 y [M, N]."""
-    if a.dtype != torch.bfloat16 or w.dtype != torch.bfloat16 or a.dim() != 2 or a.stride(1) != 1:
-        raise ValueError("a, w: bf16 matrices with unit column stride")
+def _gemm16(name: str, dtype, a: torch.Tensor, w: torch.Tensor, y, stream):
+    if a.dtype != dtype or w.dtype != dtype or a.dim() != 2 or a.stride(1) != 1:
+        raise ValueError(f"a, w: {dtype} matrices with unit column stride")
     w = w.contiguous()
     M, K = a.shape
     N = w.shape[0]
     if y is None:
-        y = torch.empty((M, N), dtype=torch.bfloat16, device=a.device)
-    _check(load_library().qlin_gemm_bf16(_ptr(a), a.stride(0), _ptr(w), M, N, K, _ptr(y),
-                                         _stream(stream)), "qlin_gemm_bf16")
+        y = torch.empty((M, N), dtype=dtype, device=a.device)
+    elif y.dtype != dtype or not y.is_contiguous() or tuple(y.shape) != (M, N):
+        raise ValueError(f"y: contiguous {dtype} [{M}, {N}]")
+    _check(getattr(load_library(), name)(_ptr(a), a.stride(0), _ptr(w), M, N, K, _ptr(y),
+                                         _stream(stream)), name)
     return y
+
+
+def qlin_gemm_bf16(a: torch.Tensor, w: torch.Tensor, y: torch.Tensor | None = None, stream=None):
+    """y = a w^T for bf16 a [M, K] (rows may be strided: any view with unit
+    column stride) and w [N, K]; bf16 y [M, N]."""
+    return _gemm16("qlin_gemm_bf16", torch.bfloat16, a, w, y, stream)
+
+
+def qlin_gemm_fp16(a: torch.Tensor, w: torch.Tensor, y: torch.Tensor | None = None, stream=None):
+    """As qlin_gemm_bf16 with fp16 operands and an fp16 y."""
+    return _gemm16("qlin_gemm_fp16", torch.float16, a, w, y, stream)
 
 
 def qlin_linear_dynamic(A: NVFP4Tensor, W: NVFP4Tensor, y: torch.Tensor | None = None,

@@ -90,6 +90,10 @@ def test_argument_errors_return_before_launch(lib):
     assert lib.qlin_gemm_bf16(16, 96, 16, 128, 128, 96, 16, None) == 1
     assert lib.qlin_gemm_bf16(16, 64, 16, 128, 128, 128, 16, None) == 1
     assert lib.qlin_gemm_bf16(16, 132, 16, 128, 128, 128, 16, None) == 3
+    # the fp16 linear shares the checks
+    assert lib.qlin_gemm_fp16(None, 128, 16, 128, 128, 128, 16, None) == 1
+    assert lib.qlin_gemm_fp16(16, 96, 16, 128, 128, 96, 16, None) == 1
+    assert lib.qlin_gemm_fp16(16, 132, 16, 128, 128, 128, 16, None) == 3
     # FP8: per-channel activation descriptor is rejected; unknown weight format
     f = qlin.FP8Desc(16, 16, 128, 256, 1)
     assert lib.qlin_quantize_act_fp8(16, 128, 256, 16, ctypes.byref(f), None, 0, None) == 1
