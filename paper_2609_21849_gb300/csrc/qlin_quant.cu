@@ -202,10 +202,13 @@ struct Fp8Op {
 
 // Persistent tile loop: thread 0 keeps kStages bulk copies of 16 KB tiles in
 // flight; every thread applies `op` to its chunks of each landed tile.
+// `setup(op)` runs once the first copies are on their way (reads that only
+// the arithmetic needs, such as the tensor scale, overlap the loads).
 // Returns false if a bounded wait expired (recorded in *err).
-template <typename Op>
+template <typename Op, typename Setup>
 __device__ __forceinline__ bool stream_tiles(const uint4* __restrict__ x, uint64_t n_chunks,
-                                             Op& op, unsigned* err, uint64_t timeout_ns) {
+                                             Op& op, Setup setup, unsigned* err,
+                                             uint64_t timeout_ns) {
   extern __shared__ __align__(128) uint8_t qsm[];
   uint4* buf = reinterpret_cast<uint4*>(qsm);
   uint64_t* full = reinterpret_cast<uint64_t*>(qsm + kStages * kTileChunks * 16);
@@ -225,14 +228,14 @@ __device__ __forceinline__ bool stream_tiles(const uint4* __restrict__ x, uint64
     for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
     abort_flag = 0;
     mbar_fence_init();
-  }
-  op.init();
-  __syncthreads();
-  if (tid == 0)
     for (int s = 0; s < kStages; ++s) {
       const uint64_t t = blockIdx.x + (uint64_t)s * gridDim.x;
       if (t < n_tiles) issue(t, s);
     }
+  }
+  setup(op);
+  op.init();
+  __syncthreads();
   int s = 0;
   uint32_t phase = 0;
   bool ok = true;
@@ -299,7 +302,7 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
   grid_dep_launch();
   __shared__ uint32_t warp_max[kThreads / 32];
   AmaxOp op;
-  stream_tiles(x, n_chunks, op, err, timeout_ns);
+  stream_tiles(x, n_chunks, op, [](AmaxOp&) {}, err, timeout_ns);
   const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, op.m);
   if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
   __syncthreads();
@@ -337,12 +340,16 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
   __shared__ float r_table[128];
   Nvfp4Op<Idx> op;
   op.r_table = r_table;
-  op.s_enc = encode_scale(tensor_scale<kDynamic>(scale_src, sdec_out, 2688.0f));
   op.chunks_per_row = (Idx)(K >> 3);
   op.K = K;
   op.codes = codes;
   op.scales = scales;
-  stream_tiles(x, n_chunks, op, err, timeout_ns);
+  stream_tiles(
+      x, n_chunks, op,
+      [&](Nvfp4Op<Idx>& o) {
+        o.s_enc = encode_scale(tensor_scale<kDynamic>(scale_src, sdec_out, 2688.0f));
+      },
+      err, timeout_ns);
 }
 
 template <bool kDynamic>
@@ -353,9 +360,11 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
   grid_dep_wait();
   grid_dep_launch();
   Fp8Op op;
-  op.s_enc = encode_scale(tensor_scale<kDynamic>(scale_src, sdec_out, 448.0f));
   op.codes = codes;
-  stream_tiles(x, n_chunks, op, err, timeout_ns);
+  stream_tiles(
+      x, n_chunks, op,
+      [&](Fp8Op& o) { o.s_enc = encode_scale(tensor_scale<kDynamic>(scale_src, sdec_out, 448.0f)); },
+      err, timeout_ns);
 }
 
 // FP8 weights, one scale per row: one warp per row, two passes over the row
