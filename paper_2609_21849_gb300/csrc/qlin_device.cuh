@@ -566,11 +566,38 @@ __device__ __forceinline__ float encode_scale(float s_dec) {
   return isinf(s) ? FLT_MAX : s;
 }
 
+// E4M3 code of the fp32 quotient t / 6 (t >= 0 or NaN).  The quotient comes
+// from the product with RN(1/6) and one fused correction step (division by a
+// divisor known in advance: Brisebarre, Muller and Raina, IEEE Trans.
+// Computers 53(8), 2004).  Its fp32 bits can differ from the correctly
+// rounded quotient only where that quotient is subnormal, and its E4M3 code
+// equals that of the correctly rounded quotient for every fp32 t in
+// [0, 4096] (an exhaustive comparison, kept as a GPU test).  Above 4096 both
+// saturate to 448, so t is clamped there first; a NaN passes through.
+__device__ __forceinline__ uint32_t e4m3_code_div6(float t) {
+  const float c = __uint_as_float(0x3E2AAAABu);   // RN(1/6)
+  const float tc = t > 4096.0f ? 4096.0f : t;
+  const float q = __fmul_rn(tc, c);
+  const float r = __fmaf_rn(-q, 6.0f, tc);
+  return e4m3_code(__fmaf_rn(r, c, q));
+}
+
+// (a, b) *= s as one packed fp32x2 multiply (each product rounded once).
+__device__ __forceinline__ void mul2_rn(float& a, float& b, float s) {
+  asm("{\n\t.reg .b64 x, y, r;\n\t"
+      "mov.b64 x, {%2, %3};\n\t"
+      "mov.b64 y, {%4, %4};\n\t"
+      "mul.rn.f32x2 r, x, y;\n\t"
+      "mov.b64 {%0, %1}, r;\n\t}"
+      : "=f"(a), "=f"(b)
+      : "f"(a), "f"(b), "f"(s));
+}
+
 // Block scale code s_b = E4M3((amax_b * S_enc) / 6) and the element
 // multiplier r_b = s_b == 0 ? 0 : S_enc / s_b (fp32, each op rounded once).
 __device__ __forceinline__ uint32_t nvfp4_block_scale(float amax_b, float s_enc, float* r_b) {
   const float t = __fmul_rn(amax_b, s_enc);
-  const uint32_t sb = e4m3_code(__fdiv_rn(t, 6.0f));
+  const uint32_t sb = e4m3_code_div6(t);
   *r_b = (sb == 0u) ? 0.0f : __fdiv_rn(s_enc, e4m3_value(sb));
   return sb;
 }

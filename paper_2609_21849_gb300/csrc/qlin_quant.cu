@@ -70,6 +70,7 @@ struct AmaxOp {
 template <typename Idx>
 struct Nvfp4Op {
   static constexpr int kUnit = 2;
+  static constexpr bool kBlockMax = true;   // the one-read kernel keeps block maxima
   float s_enc;
   Idx chunks_per_row;
   int64_t K;
@@ -83,22 +84,23 @@ struct Nvfp4Op {
       r_table[c] = (c == 0u) ? 0.0f : __fdiv_rn(s_enc, e4m3_value(c));
     }
   }
-  // The codes of one 16-element block and its scale code; lanes 4g..4g+3
-  // hold one 64-element group, whose four scales are gathered into lane 4g.
-  __device__ __forceinline__ void quantize_block(const uint4 (&v)[2], uint32_t& code0,
-                                                 uint32_t& code1, uint32_t& word) const {
-    const uint32_t mb = max(chunk_abs_max_bits(v[0]), chunk_abs_max_bits(v[1]));
+  // The codes of one 16-element block (block amax bits mb) and its scale
+  // code; lanes 4g..4g+3 hold one 64-element group, whose four scales are
+  // gathered into lane 4g.
+  __device__ __forceinline__ void quantize_block(const uint4 (&v)[2], uint32_t mb,
+                                                 uint32_t& code0, uint32_t& code1,
+                                                 uint32_t& word) const {
     const float t = __fmul_rn(__uint_as_float(mb << 16), s_enc);
-    const uint32_t sb = e4m3_code(__fdiv_rn(t, 6.0f));
+    const uint32_t sb = e4m3_code_div6(t);
     const float r_b = r_table[sb];
     float f[8];
     unpack8(v[0], f);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], r_b);
+    for (int i = 0; i < 8; i += 2) mul2_rn(f[i], f[i + 1], r_b);
     code0 = e2m1x8(f);
     unpack8(v[1], f);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) f[i] = __fmul_rn(f[i], r_b);
+    for (int i = 0; i < 8; i += 2) mul2_rn(f[i], f[i + 1], r_b);
     code1 = e2m1x8(f);
     const uint32_t s1 = __shfl_down_sync(0xFFFFFFFFu, sb, 1);
     const uint32_t s2 = __shfl_down_sync(0xFFFFFFFFu, sb, 2);
@@ -107,7 +109,8 @@ struct Nvfp4Op {
   }
   __device__ __forceinline__ void unit(const uint4 (&v)[2], uint64_t c, bool valid) {
     uint32_t code0, code1, word;
-    quantize_block(v, code0, code1, word);
+    quantize_block(v, max(chunk_abs_max_bits(v[0]), chunk_abs_max_bits(v[1])), code0, code1,
+                   word);
     if (valid) {
       reinterpret_cast<uint2*>(codes)[c >> 1] = make_uint2(code0, code1);
       if ((threadIdx.x & 3) == 0) {
@@ -122,9 +125,12 @@ struct Nvfp4Op {
   // A slice of n chunks held in shared memory, global chunks [c0, c0 + n)
   // (c0 and n multiples of 8): each thread takes units of two chunks at a
   // stride of the block, two units per step for instruction-level
-  // parallelism, and tracks its row and column without dividing.
-  template <int kThreadsPerBlock>
-  __device__ __forceinline__ void run_slice(const uint4* buf, uint32_t n, uint64_t c0) const {
+  // parallelism, and tracks its row and column without dividing.  The
+  // block amax bits of step s's two units are bm[s] (low, high halves), as
+  // gathered by block_max_pass.
+  template <int kThreadsPerBlock, int kSteps>
+  __device__ __forceinline__ void run_slice(const uint4* buf, uint32_t n, uint64_t c0,
+                                            const uint32_t (&bm)[kSteps]) const {
     constexpr uint32_t kStride = 2u * kThreadsPerBlock;          // chunks per step and unit
     const uint32_t cpr = (uint32_t)chunks_per_row;
     const uint32_t dq = (2u * kStride) / cpr, dr = (2u * kStride) % cpr;
@@ -133,7 +139,10 @@ struct Nvfp4Op {
     uint32_t row = (uint32_t)(cg / cpr), col = (uint32_t)(cg % cpr);   // col in chunks
     const uint32_t kgroups = (uint32_t)(K >> 6);
     // the loop bound is block-uniform: every lane reaches the shuffles
-    for (uint32_t base = 0; base < n; base += 2u * kStride) {
+#pragma unroll
+    for (int s = 0; s < kSteps; ++s) {
+      const uint32_t base = (uint32_t)s * 2u * kStride;
+      if (base >= n) break;
       const uint32_t cl = base + 2u * threadIdx.x;
       uint4 va[2], vb[2];
       const bool ok_a = cl < n, ok_b = cl + kStride < n;   // units never straddle n
@@ -143,8 +152,8 @@ struct Nvfp4Op {
         vb[k] = ok_b ? lds128(buf + cl + kStride + k) : make_uint4(0u, 0u, 0u, 0u);
       }
       uint32_t a0, a1, aw, b0, b1, bw;
-      quantize_block(va, a0, a1, aw);
-      quantize_block(vb, b0, b1, bw);
+      quantize_block(va, bm[s] & 0xFFFFu, a0, a1, aw);
+      quantize_block(vb, bm[s] >> 16, b0, b1, bw);
       uint32_t row_b = row + kq, col_b = col + kr;
       if (col_b >= cpr) {
         col_b -= cpr;
@@ -175,6 +184,7 @@ struct Nvfp4Op {
 
 struct Fp8Op {
   static constexpr int kUnit = 1;
+  static constexpr bool kBlockMax = false;
   float s_enc;
   uint2* codes;
   __device__ __forceinline__ void bind(float*) {}
@@ -409,6 +419,8 @@ __global__ void __launch_bounds__(kThreads) quant_fp8_rows_kernel(const uint4* _
 constexpr int kOnePassThreads = 1024;
 constexpr int kOnePassSmem = 225 * 1024;
 constexpr int kOnePassSliceMax = 14 * 1024;       // chunks: 224 KB of data at most
+// NVFP4 steps of run_slice: two 2-chunk units per thread and step
+constexpr int kOnePassSteps = (kOnePassSliceMax + 4 * kOnePassThreads - 1) / (4 * kOnePassThreads);
 
 __device__ __forceinline__ uint32_t ld_acquire_gpu(const unsigned* p) {
   uint32_t v;
@@ -440,13 +452,46 @@ __global__ void __launch_bounds__(kOnePassThreads, 1)
   const uint32_t n = c_begin >= n_chunks ? 0u
                      : (uint32_t)(n_chunks - c_begin < slice ? n_chunks - c_begin : slice);
   // every thread copies its chunks (a dozen 16-byte asynchronous copies in
-  // flight per thread), then takes their amax
+  // flight per thread), then takes their amax; it reads only the chunks it
+  // copied itself, so waiting for its own copies suffices.  NVFP4 copies in
+  // the units run_slice quantizes (two adjacent chunks, a warp covering 1 KB)
   const uint4* xs = x + c_begin;
-  for (uint32_t i = tid; i < n; i += kOnePassThreads) cp_async16(smem_u32(buf + i), xs + i);
+  if constexpr (Op::kBlockMax) {
+#pragma unroll
+    for (int s = 0; s < 2 * kOnePassSteps; ++s) {
+      const uint32_t c = (uint32_t)s * 2u * kOnePassThreads + 2u * tid;
+      if (c < n) {
+        cp_async16(smem_u32(buf + c), xs + c);
+        cp_async16(smem_u32(buf + c + 1), xs + c + 1);
+      }
+    }
+  } else {
+    for (uint32_t i = tid; i < n; i += kOnePassThreads) cp_async16(smem_u32(buf + i), xs + i);
+  }
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
   grid_dep_launch();   // x is on chip: the next kernel may begin launching
   uint32_t m = 0;
-  for (uint32_t i = tid; i < n; i += kOnePassThreads) m = max(m, chunk_abs_max_bits(lds128(buf + i)));
+  uint32_t bm[kOnePassSteps] = {};
+  if constexpr (Op::kBlockMax) {
+    // NVFP4: the amax of each 16-element block this thread will quantize
+    // (the units of run_slice), kept for after the barrier
+#pragma unroll
+    for (int s = 0; s < kOnePassSteps; ++s) {
+      const uint32_t ca = (uint32_t)s * 4u * kOnePassThreads + 2u * tid;
+      const uint32_t cb = ca + 2u * kOnePassThreads;
+      const uint32_t a =
+          ca < n ? max(chunk_abs_max_bits(lds128(buf + ca)), chunk_abs_max_bits(lds128(buf + ca + 1)))
+                 : 0u;
+      const uint32_t b =
+          cb < n ? max(chunk_abs_max_bits(lds128(buf + cb)), chunk_abs_max_bits(lds128(buf + cb + 1)))
+                 : 0u;
+      bm[s] = a | (b << 16);
+      m = max(m, max(a, b));
+    }
+  } else {
+    for (uint32_t i = tid; i < n; i += kOnePassThreads)
+      m = max(m, chunk_abs_max_bits(lds128(buf + i)));
+  }
   m = __reduce_max_sync(0xFFFFFFFFu, m);
   if ((tid & 31) == 0) warp_max[tid >> 5] = m;
   if (tid == 0) abort_flag = 0;
@@ -484,7 +529,10 @@ __global__ void __launch_bounds__(kOnePassThreads, 1)
   op.bind(op_table);
   op.init();
   __syncthreads();
-  op.template run_slice<kOnePassThreads>(buf, n, c_begin);
+  if constexpr (Op::kBlockMax)
+    op.template run_slice<kOnePassThreads, kOnePassSteps>(buf, n, c_begin, bm);
+  else
+    op.template run_slice<kOnePassThreads>(buf, n, c_begin);
 }
 
 // Opt each kernel into kSmem bytes of dynamic shared memory, once.
