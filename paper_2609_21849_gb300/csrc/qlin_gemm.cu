@@ -75,8 +75,12 @@ struct Cfg {
   static constexpr int kSfaBytes = kFp4 ? kStepsPerStage * 512 : 0;
   static constexpr int kSfbBytes = kFp4 ? kSfbAtoms * kStepsPerStage * 512 : 0;
   static constexpr int kStageBytes = kABytes + kBBytes + kSfaBytes + kSfbBytes;
-  // epilogue staging: per epilogue warp two 32 x 32 bf16 boxes (2 KB each)
-  static constexpr int kOutBytes = kEpiWarps * 2 * 2048;
+  // FP8 / 16-bit pair tiles store y straight from registers (each thread
+  // its row's 64 bytes per 32 columns), which frees the staging boxes for a
+  // seventh pipeline stage; otherwise per epilogue warp two 32 x 32 bf16
+  // boxes (2 KB each) stage TMA stores
+  static constexpr bool kDirectStore = !kFp4 && kPair && kBN == 256;
+  static constexpr int kOutBytes = kDirectStore ? 0 : kEpiWarps * 2 * 2048;
   static constexpr int kStagesRaw = (kSmemBudget - kOutBytes) / kStageBytes;
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
   static constexpr int kNumAcc = (kFp4 && kBN == 256) ? 1 : 2;
@@ -107,6 +111,7 @@ struct KParams {
   int64_t rq_col0, rq_cols;
   unsigned* y_amax;   // optional: max |bf16 y| over the output, as fp32 bits (atomicMax)
   int fp16;           // 16-bit operand kernel only: fp16 operands and output (else bf16)
+  int y_v8;           // y is 32-byte aligned: direct stores may use 32-byte vectors
   unsigned* err;
   uint64_t timeout_ns;
 };
@@ -129,6 +134,13 @@ __device__ __forceinline__ void st_global_v4(void* p, uint32_t a, uint32_t b, ui
                                              uint32_t d) {
   asm volatile("st.global.v4.b32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(a), "r"(b), "r"(c),
                "r"(d)
+               : "memory");
+}
+
+// 32-byte store (p 32-byte aligned): a whole L2 sector from one lane.
+__device__ __forceinline__ void st_global_v8(void* p, const uint32_t* v) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(v[0]),
+               "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
                : "memory");
 }
 
@@ -463,7 +475,6 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
     const int e = warp - C::kEpiWarp0;
     const int quarter = warp & 3;   // the TMEM lane quarter this warp may access
     const int half = e >> 2;
-    uint8_t* const out_buf = out_stage + e * 4096;   // this warp's two staging boxes
     const float sdec_a = kBf16 ? 1.0f : *p.sdec_a;
     const float alpha = kFp4 ? __fmul_rn(sdec_a, *p.sdec_w) : kBf16 ? 1.0f : 0.0f;
     float s_enc_next = 0.0f;
@@ -565,9 +576,31 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
         m = __reduce_max_sync(0xFFFFFFFFu, m);
         if (lane == 0 && m != 0u) atomicMax(p.y_amax, m << 16);
       }
-      if (p.y != nullptr) {
+      if constexpr (C::kDirectStore) {
+        // 16-bit output straight from registers: the thread's row, 32
+        // columns (64 bytes) per chunk; N % 64 == 0, so a chunk is wholly
+        // inside or outside the matrix
+        if (p.y != nullptr && row < p.M) {
+          uint16_t* const yrow = p.y + row * p.N + col0;
+#pragma unroll
+          for (int c = 0; c < kChunks; ++c) {
+            if (col0 + c * 32 >= p.N) break;
+            uint32_t* const dst = reinterpret_cast<uint32_t*>(yrow + c * 32);
+            if (p.y_v8) {
+              st_global_v8(dst, &packed[c * 16]);
+              st_global_v8(dst + 8, &packed[c * 16 + 8]);
+            } else {
+#pragma unroll
+              for (int k = 0; k < 4; ++k)
+                st_global_v4(dst + 4 * k, packed[c * 16 + 4 * k], packed[c * 16 + 4 * k + 1],
+                             packed[c * 16 + 4 * k + 2], packed[c * 16 + 4 * k + 3]);
+            }
+          }
+        }
+      } else if (p.y != nullptr) {
         // bf16 output: each 32 x 32 box goes through a 64-byte-swizzled
         // staging buffer and one TMA store (rows >= M, cols >= N are clipped).
+        uint8_t* const out_buf = out_stage + e * 4096;   // this warp's two staging boxes
 #pragma unroll
         for (int c = 0; c < kChunks; ++c) {
           uint8_t* const bufp = out_buf + (c & 1) * 2048;
@@ -786,6 +819,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   p.rq_cols = a.rq_cols;
   p.y_amax = a.y_amax;
   p.fp16 = kBf16 && a.fp16 ? 1 : 0;
+  p.y_v8 = (reinterpret_cast<uintptr_t>(a.y) & 31u) == 0 ? 1 : 0;
   p.err = err;
   p.timeout_ns = timeout_ns;
   auto kern = gemm_kernel<kFp4, kBN, kPair, kRequant, kBf16>;

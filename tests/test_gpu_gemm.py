@@ -129,3 +129,23 @@ def test_nvfp4_dyadic_exact():
     assert np.array_equal(yref, x.astype(np.float64) @ w.astype(np.float64).T)
     err, exact = gemm_errors(bf16_bits(y), yref, na, nw)
     assert exact == 1.0, exact
+
+
+def test_fp8_output_alignment_16_and_32_bytes():
+    # The pair-tile FP8 epilogue stores y straight from registers, with
+    # 32-byte vectors when y is 32-byte aligned and 16-byte ones otherwise;
+    # both must write the same bits (rows 1..M of a padded buffer check that
+    # nothing lands outside y).
+    x, w = synthetic.fp8_linear()
+    A = qlin.qlin_quantize_act_fp8(to_dev(x))
+    W = qlin.qlin_quantize_weight(to_dev(w), qlin.QLIN_FMT_FP8)
+    M, N = A.rows, W.rows
+    y32 = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    qlin.qlin_gemm_fp8(A, W, y32)
+    pad = torch.full((M * N + 32,), -7.0, dtype=torch.bfloat16, device="cuda")
+    y16 = pad[8:8 + M * N].view(M, N)              # 16 bytes past a 32-byte boundary
+    assert y16.data_ptr() % 32 == 16
+    qlin.qlin_gemm_fp8(A, W, y16)
+    assert qlin.qlin_sync_status() == 0
+    assert torch.equal(y16.view(torch.int16), y32.view(torch.int16))
+    assert torch.all(pad[:8] == -7.0) and torch.all(pad[8 + M * N:] == -7.0)
