@@ -1,6 +1,6 @@
 """GPU parity of the denoise-step linear stack (8 blocks x QKV / out / up /
-down, NVFP4 W4A4, chained fused re-quantization), batch 1 (M = 4608), in the
-launch configuration the benchmark times.
+down, NVFP4 W4A4, chained fused re-quantization), batch 1 and 4 (M = 4608,
+18432), in the launch configuration the benchmark times.
 
 The oracle runs the same chain on a few sampled token rows (every layer is
 row-local once its static input scale is fixed): exact fp64 GEMM, its own bf16
@@ -21,11 +21,25 @@ if torch.cuda.is_available():
                           requant_agreement, sample_rows, to_dev)
 
 
-def test_stack_b1_chain():
-    M = synthetic.M_TOKENS
-    R = sample_rows(M, 6, seed=9)
-    x = synthetic.stack_input(1)
-    wlist = list(synthetic.stack_weights(8, 4))
+_WEIGHTS = {}
+
+
+def _weights():
+    """The stack's seeded weights and the oracle's quantization of them
+    (shared by the batch sizes)."""
+    if not _WEIGHTS:
+        wlist = list(synthetic.stack_weights(8, 4))
+        _WEIGHTS["w"] = wlist
+        _WEIGHTS["q"] = [oracle.quant_nvfp4(w) for (_, _, w) in wlist]
+    return _WEIGHTS["w"], _WEIGHTS["q"]
+
+
+@pytest.mark.parametrize("B", [1, 4])
+def test_stack_chain(B):
+    M = synthetic.M_TOKENS * B
+    R = sample_rows(M, 6, seed=9 + B)
+    x = synthetic.stack_input(B)
+    wlist, wqs = _weights()
 
     # ---- oracle chain on the sampled rows
     s0 = oracle.nvfp4_tensor_scale(oracle.amax_bf16(x))
@@ -33,7 +47,7 @@ def test_stack_b1_chain():
     a0_ref = a_rows
     refs, wq0 = [], None
     for i, (b, name, w) in enumerate(wlist):
-        wq = oracle.quant_nvfp4(w)
+        wq = wqs[i]
         if i < 4:
             wq0 = (wq0 or []) + [wq]
         yref, na, nw = oracle.gemm_nvfp4(a_rows, wq)
@@ -45,7 +59,7 @@ def test_stack_b1_chain():
         a_rows = oracle.quant_nvfp4(win, s_next)
 
     # ---- GPU: all rows, same weights and static scales
-    st = stack.build_stack(1, weights=wlist)
+    st = stack.build_stack(B, weights=wlist)
     st.set_next_scales([r[4] for r in refs])
     st.forward(to_dev(x))
     assert qlin.qlin_sync_status() == 0
@@ -68,4 +82,4 @@ def test_stack_b1_chain():
         agree = requant_agreement(codes[R], canon[R], np.ascontiguousarray(yb[:, c0:]), win, s_next)
         assert agree >= 0.99, (i, agree)
         worst, agree_min = max(worst, err.max()), min(agree_min, agree)
-    print(f"stack B=1: worst normalised error {worst:.2e}, min requant agreement {agree_min:.5f}")
+    print(f"stack B={B}: worst normalised error {worst:.2e}, min requant agreement {agree_min:.5f}")
