@@ -666,8 +666,9 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
                 float f[8];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                  f[2 * i] = __fmul_rn(bf16_lo(pk[h8 * 4 + i]), r_b);
-                  f[2 * i + 1] = __fmul_rn(bf16_hi(pk[h8 * 4 + i]), r_b);
+                  f[2 * i] = bf16_lo(pk[h8 * 4 + i]);
+                  f[2 * i + 1] = bf16_hi(pk[h8 * 4 + i]);
+                  mul2_rn(f[2 * i], f[2 * i + 1], r_b);
                 }
                 words[b * 2 + h8] = e2m1x8(f);
               }
