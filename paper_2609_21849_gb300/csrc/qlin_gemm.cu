@@ -1,8 +1,10 @@
 // Block-scaled GEMMs on the 5th-generation tensor cores (tcgen05) of sm_103a:
 // the NVFP4 and FP8 linear layers of Sec. 4 ("Quantization": activation
 // quantization lets the linears run on the FP8 / NVFP4 tensor cores), with a
-// fused epilogue that writes the bf16 output and, optionally, re-quantizes it
-// to NVFP4 for the next layer.
+// fused epilogue that writes the 16-bit output and, optionally, re-quantizes
+// it for the next layer (NVFP4 or FP8) or reduces its tensor amax.  The same
+// skeleton runs the unquantized bf16 / fp16 linears of Table 2's precision
+// ladder (kind::f16).
 //
 // Two tile configurations share one kernel template:
 //   pair   256 x 256 output tiles on a CTA pair (a cluster of two CTAs on two
@@ -10,19 +12,25 @@
 //          drives both SMs' tensor cores; each CTA holds its own 128 rows of A
 //          and its own half of the W tile in shared memory.
 //   single 128 x 128 tiles on one CTA, for small M (the translator's linears).
-// Roles (one persistent CTA per SM; 12 warps, 14 for NVFP4 pair tiles):
-//   warp 0      TMA producer: per pipeline stage one 4-D tensor copy per lane
-//               (A tile, W tile, A scale atoms, W scale atoms), issued by four
-//               lanes as a single instruction.  In a pair, CTA 1's copies
-//               complete on CTA 0's barriers (cta_group::2 form).
+// Roles (one persistent CTA per SM; 12 warps, 13 for NVFP4 pair tiles):
+//   warp 0      TMA producer: per pipeline stage one 4-D tensor copy per lane,
+//               the A tile and the W tile from two lanes as one instruction
+//               (and, except for NVFP4 pair tiles, the A and W scale atoms
+//               from two more lanes).  In a pair, CTA 1's copies complete on
+//               CTA 0's barriers (cta_group::2 form).
 //   warp 1      TMEM allocation; MMA issue (per 32 bytes of K one tcgen05.mma:
 //               NVFP4 kind::mxf4nvf4 scale_vec::4X with K = 64, FP8
-//               kind::f8f6f4 with K = 32) into an fp32 TMEM accumulator.
-//   warps 2..   NVFP4: block scales shared -> TMEM (tcgen05.cp), beside the
-//               MMA stream (two warps, four for pair tiles).
-//   last 8      epilogue: tcgen05.ld of the accumulator, alpha, bf16, TMA
-//               stores through swizzled staging, optional NVFP4 re-quantization
-//               of the bf16 values (one row per thread).
+//               kind::f8f6f4 with K = 32, bf16 / fp16 kind::f16 with K = 16)
+//               into an fp32 TMEM accumulator.
+//   warps 2, 3  NVFP4: block scales shared -> TMEM (tcgen05.cp), beside the
+//               MMA stream, each warp the atoms of half the stage's MMA steps.
+//   warp 4      NVFP4 pair tiles: TMA producer of the scale atoms.
+//   last 8      epilogue: tcgen05.ld of the accumulator, alpha, 16-bit
+//               rounding; NVFP4 tiles store y by TMA through swizzled staging,
+//               FP8 / 16-bit pair tiles store it straight from registers (the
+//               staging's shared memory holds a seventh stage instead);
+//               optional re-quantization of the 16-bit values, one row per
+//               thread, and optional output amax.
 // Every wait is bounded (see WaitCtl).
 #include <cstring>
 #include <mutex>
@@ -37,16 +45,19 @@ constexpr int kBM = 128;
 constexpr int kRowBytes = 128;      // bytes of K per stage and row: one swizzle row
 constexpr int kStepsPerStage = 4;   // one MMA per 32 bytes of K
 constexpr int kEpiWarps = 8;
+// Build-time layout choices (the defaults measured fastest): scale-copy warps
+// of NVFP4 pair tiles, a warp of its own for their scale boxes, and row boxes
+// per operand tile and stage.
 #ifndef QLIN_PAIR_CP_WARPS
 #define QLIN_PAIR_CP_WARPS 2
 #endif
 #ifndef QLIN_SPLIT_SCALE_ISSUE
 #define QLIN_SPLIT_SCALE_ISSUE 1
 #endif
-constexpr int kSmemBudget = 232448 - 2048;  // opt-in shared memory minus barriers/alignment
 #ifndef QLIN_TMA_SPLIT
 #define QLIN_TMA_SPLIT 1
 #endif
+constexpr int kSmemBudget = 232448 - 2048;  // opt-in shared memory minus barriers/alignment
 constexpr int kSplit = QLIN_TMA_SPLIT;      // row boxes per operand tile and stage
 
 constexpr int pow2_at_least(int x) {
@@ -62,7 +73,7 @@ struct Cfg {
   // warps: 0 producer, 1 MMA, then the scale-copy warps, then the epilogue
   // (an epilogue warp w reads TMEM lanes 32 (w % 4) and up, so any eight
   // consecutive warps cover the accumulator).  NVFP4 pair tiles need 12
-  // scale copies per stage, more than two warps issue in an MMA stage.
+  // scale copies per stage, shared between the scale-copy warps.
   static constexpr int kCpWarps = (kFp4 && kPair) ? QLIN_PAIR_CP_WARPS : 2;
   // NVFP4 pair tiles: a warp of its own issues the scale boxes, so the
   // operand boxes' instruction has two lanes instead of four
