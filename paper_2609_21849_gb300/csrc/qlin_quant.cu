@@ -513,14 +513,17 @@ __global__ void __launch_bounds__(kOnePassThreads, 1)
       }
     }
     s_amax = __uint_as_float(ld_acquire_gpu(&sync[0]));
-    // depart (after a timeout too); the last CTA out resets the words
+  }
+  __syncthreads();
+  if (tid == 0) {
+    // depart (after a timeout too); the last CTA out resets the words.  The
+    // other warps do not wait for this atomic's round trip.
     if (atomicAdd(&sync[2], 1u) == gridDim.x - 1u) {
       sync[0] = 0u;
       sync[1] = 0u;
       sync[2] = 0u;
     }
   }
-  __syncthreads();
   if (abort_flag) return;
   const float amax = s_amax;
   const float s_dec = (amax == 0.0f) ? 1.0f : __fdiv_rn(amax, qmax);
