@@ -73,6 +73,10 @@ struct Nvfp4Op {
   static constexpr bool kBlockMax = true;   // the one-read kernel keeps block maxima
   float s_enc;
   Idx chunks_per_row;
+  // row = chunk / chunks_per_row without a division (32-bit indices):
+  // t = umulhi(div_m, c), row = (t + ((c - t) >> div_s1)) >> div_s2
+  // (Granlund and Montgomery, PLDI 1994, division by invariant integers)
+  uint32_t div_m, div_s1, div_s2;
   int64_t K;
   uint32_t* codes;
   uint8_t* scales;
@@ -114,11 +118,20 @@ struct Nvfp4Op {
     if (valid) {
       reinterpret_cast<uint2*>(codes)[c >> 1] = make_uint2(code0, code1);
       if ((threadIdx.x & 3) == 0) {
-        const Idx ci = (Idx)c;
-        const Idx row = ci / chunks_per_row;
-        const Idx col = (ci - row * chunks_per_row) << 3;
-        *reinterpret_cast<uint32_t*>(scales + scale_offset((int64_t)row, (int64_t)(col >> 4), K)) =
-            word;
+        if constexpr (sizeof(Idx) == 4) {
+          const uint32_t ci = (uint32_t)c;
+          const uint32_t t = __umulhi(div_m, ci);
+          const uint32_t row = (t + ((ci - t) >> div_s1)) >> div_s2;
+          const uint32_t colc = ci - row * (uint32_t)chunks_per_row;   // in chunks
+          *reinterpret_cast<uint32_t*>(scales + ((row >> 7) * (uint32_t)(K >> 6) + (colc >> 3)) * 512u +
+                                       (row & 31u) * 16u + ((row >> 5) & 3u) * 4u) = word;
+        } else {
+          const Idx ci = (Idx)c;
+          const Idx row = ci / chunks_per_row;
+          const Idx col = (ci - row * chunks_per_row) << 3;
+          *reinterpret_cast<uint32_t*>(scales + scale_offset((int64_t)row, (int64_t)(col >> 4), K)) =
+              word;
+        }
       }
     }
   }
@@ -344,13 +357,17 @@ template <bool kDynamic, typename Idx>
 __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
     quant_nvfp4_kernel(const uint4* __restrict__ x, uint64_t n_chunks, int64_t K,
                        const float* scale_src, float* sdec_out, uint32_t* __restrict__ codes,
-                       uint8_t* __restrict__ scales, unsigned* err, uint64_t timeout_ns) {
+                       uint8_t* __restrict__ scales, uint3 row_div, unsigned* err,
+                       uint64_t timeout_ns) {
   grid_dep_wait();
   grid_dep_launch();
   __shared__ float r_table[128];
   Nvfp4Op<Idx> op;
   op.r_table = r_table;
   op.chunks_per_row = (Idx)(K >> 3);
+  op.div_m = row_div.x;
+  op.div_s1 = row_div.y;
+  op.div_s2 = row_div.z;
   op.K = K;
   op.codes = codes;
   op.scales = scales;
@@ -645,6 +662,7 @@ cudaError_t launch_quant_nvfp4_onepass(const void* x, int64_t M, int64_t K,
   Nvfp4Op<uint32_t> op;
   op.s_enc = 0.0f;   // set in the kernel once amax is known
   op.chunks_per_row = (uint32_t)(K >> 3);
+  op.div_m = op.div_s1 = op.div_s2 = 0;   // run_slice tracks rows without dividing
   op.K = K;
   op.codes = reinterpret_cast<uint32_t*>(out.codes);
   op.scales = out.scales;
@@ -664,11 +682,22 @@ cudaError_t launch_quant_fp8_onepass(const void* x, int64_t M, int64_t K, const 
                         timeout_ns);
 }
 
+// Multiplier and shifts that divide a 32-bit index by d (1 <= d < 2^31)
+// without a division instruction: the round-up form of Granlund and
+// Montgomery (PLDI 1994), exact for every 32-bit dividend.
+static uint3 invariant_divisor(uint32_t d) {
+  int l = 0;
+  while ((1ull << l) < d) ++l;   // ceil(log2 d)
+  const uint64_t m = ((1ull << 32) * ((1ull << l) - d)) / d + 1;
+  return make_uint3((uint32_t)m, (uint32_t)(l < 1 ? l : 1), (uint32_t)(l > 1 ? l - 1 : 0));
+}
+
 template <bool kDynamic>
 static cudaError_t launch_nvfp4_t(const void* x, int64_t M, int64_t K, const float* scale_src,
                                   const qlin_nvfp4_t& out, cudaStream_t s, int num_sms,
                                   unsigned* err, uint64_t timeout_ns) {
   const uint64_t n_chunks = (uint64_t)M * (uint64_t)K / 8;
+  const uint3 row_div = invariant_divisor((uint32_t)(K >> 3));
   const int grid = stream_grid(n_chunks, num_sms);
   auto* xin = static_cast<const uint4*>(x);
   auto* codes = reinterpret_cast<uint32_t*>(out.codes);
@@ -676,11 +705,13 @@ static cudaError_t launch_nvfp4_t(const void* x, int64_t M, int64_t K, const flo
   if (n_chunks < (1ull << 32)) {   // 32-bit index math is enough
     if ((e = set_smem<quant_nvfp4_kernel<kDynamic, uint32_t>>()) != cudaSuccess) return e;
     e = launch_pdl(quant_nvfp4_kernel<kDynamic, uint32_t>, grid, kThreads, kSmem, s, xin,
-                   n_chunks, K, scale_src, out.tensor_scale, codes, out.scales, err, timeout_ns);
+                   n_chunks, K, scale_src, out.tensor_scale, codes, out.scales, row_div, err,
+                   timeout_ns);
   } else {
     if ((e = set_smem<quant_nvfp4_kernel<kDynamic, uint64_t>>()) != cudaSuccess) return e;
     e = launch_pdl(quant_nvfp4_kernel<kDynamic, uint64_t>, grid, kThreads, kSmem, s, xin,
-                   n_chunks, K, scale_src, out.tensor_scale, codes, out.scales, err, timeout_ns);
+                   n_chunks, K, scale_src, out.tensor_scale, codes, out.scales, row_div, err,
+                   timeout_ns);
   }
   return e;
 }
