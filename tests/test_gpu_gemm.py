@@ -149,3 +149,14 @@ def test_fp8_output_alignment_16_and_32_bytes():
     assert qlin.qlin_sync_status() == 0
     assert torch.equal(y16.view(torch.int16), y32.view(torch.int16))
     assert torch.all(pad[:8] == -7.0) and torch.all(pad[8 + M * N:] == -7.0)
+
+
+def test_nvfp4_ragged_pair_tiles_partial_last_wave():
+    # 4500 x 12224 on CTA pairs: 864 tiles of 256 x 256 over the persistent
+    # clusters, a partial last wave, a partial last row block (20 rows) and a
+    # last N block with 192 valid columns of 256.
+    M, N, K = 4500, 12224, 1024
+    x = synthetic.act_entry_outliers(77, M, K)
+    (w,) = synthetic.weights(78, [(N, K)], 0.02)
+    rows = np.unique(np.concatenate([sample_rows(M, 40, seed=5), np.arange(M - 20, M)]))
+    _check_nvfp4(x, w, rows, "pair tiles 4500x12224x1024")
