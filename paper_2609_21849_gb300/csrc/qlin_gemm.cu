@@ -292,7 +292,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
             dst = sB + C::kBBytes; c0 = kb * kStepsPerStage * 64; c1 = mb; c2 = 0; c3 = 0;
           } else {                          // W scale atoms (all atom rows of the N tile)
             dst = sB + C::kBBytes + C::kSfaBytes; c0 = kb * kStepsPerStage * 64;
-            c1 = nb * C::kSfbAtoms; c2 = 0; c3 = 0;
+            c1 = (nb * kBN) >> 7; c2 = 0; c3 = 0;   // first 128-row atom of the N tile
           }
           const uint32_t bar = bar0 + (uint32_t)(stage * 8);
           if (kPair)
@@ -338,6 +338,10 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
       uint32_t acc_phase = 0;
       bool ok = true;
       for (int ct = cid; ct < num_ctiles && ok; ct += ncl) {
+        // 64-wide tiles use one half of a 128-row W scale atom: its rows
+        // 32 w + lane sit in TMEM column w, so the odd tile's half starts two
+        // columns in
+        const uint32_t sfb_off = kBN < 128 ? 2u * (uint32_t)((ct / groups_m) & 1) : 0u;
         if (!mbar_wait(&tmem_empty[acc], acc_phase ^ 1u, ctl) || !wait_ready(stage, phase)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * kBN);
@@ -355,7 +359,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
               if (kPair)
                 mma_nvfp4_pair(d_tmem, adesc, bdesc, idesc, sfa_t, sfa_t + 4, accumulate);
               else
-                mma_nvfp4(d_tmem, adesc, bdesc, idesc, sfa_t, sfa_t + 4, accumulate);
+                mma_nvfp4(d_tmem, adesc, bdesc, idesc, sfa_t, sfa_t + 4 + sfb_off, accumulate);
             } else if (kBf16) {
               if (kPair)
                 mma_bf16_pair(d_tmem, adesc, bdesc, idesc, accumulate);
@@ -512,7 +516,8 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
       // With a single accumulator the next tile's MMAs wait for that, so all
       // columns form one batch where the register budget (168 a thread at
       // 12 warps, 128 above) allows.
-      constexpr int kBatch = (C::kNumAcc == 1 && C::kThreads <= 384) ? kChunks : 2;
+      constexpr int kBatch =
+          (C::kNumAcc == 1 && C::kThreads <= 384) ? kChunks : (kChunks < 2 ? kChunks : 2);
 #pragma unroll
       for (int cb = 0; cb < kChunks; cb += kBatch) {
         uint32_t r[kBatch][32];
@@ -876,14 +881,18 @@ template <bool kFp4>
 cudaError_t dispatch_bn(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned* err,
                         uint64_t timeout_ns) {
   // 256 x 256 tiles on CTA pairs when they fill the machine, else 128 x 128
-  // single-CTA tiles (small M).
-  const int64_t tiles256 = ((a.M + kBM - 1) / kBM) * ((a.N + 255) / 256);
-  const bool wide = tiles256 >= num_sms;
+  // single-CTA tiles (small M), or 128 x 64 when 128 x 128 tiles would leave
+  // at least half the SMs idle (no fused re-quantization: its 64-column
+  // groups need 128-column tiles).
+  const int64_t tiles_m = (a.M + kBM - 1) / kBM;
+  const bool wide = tiles_m * ((a.N + 255) / 256) >= num_sms;
   if (a.next_scale != nullptr)
     return wide ? launch_cfg<kFp4, 256, true, true>(a, s, num_sms, err, timeout_ns)
                 : launch_cfg<kFp4, 128, false, true>(a, s, num_sms, err, timeout_ns);
-  return wide ? launch_cfg<kFp4, 256, true, false>(a, s, num_sms, err, timeout_ns)
-              : launch_cfg<kFp4, 128, false, false>(a, s, num_sms, err, timeout_ns);
+  if (wide) return launch_cfg<kFp4, 256, true, false>(a, s, num_sms, err, timeout_ns);
+  const bool narrow = 2 * tiles_m * ((a.N + 127) / 128) <= num_sms;
+  return narrow ? launch_cfg<kFp4, 64, false, false>(a, s, num_sms, err, timeout_ns)
+                : launch_cfg<kFp4, 128, false, false>(a, s, num_sms, err, timeout_ns);
 }
 
 }  // namespace
