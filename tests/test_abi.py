@@ -110,3 +110,25 @@ def test_python_binding_fails_loudly_without_library(tmp_path):
             qlin.load_library(str(tmp_path / "missing.so"))
     finally:
         qlin._lib = saved
+
+
+def test_empty_dimensions_are_rejected_before_launch(lib):
+    # an empty matrix (M, N or K of 0) has nothing to compute; every entry
+    # point reports it as an argument error instead of launching
+    from paper_2609_21849_gb300 import qlin
+    d0 = qlin.NVFP4Desc(16, 16, 16, 0, 256)
+    assert lib.qlin_quantize_act_nvfp4(16, 0, 256, 16, ctypes.byref(d0), 16, 256, None) == 1
+    dk = qlin.NVFP4Desc(16, 16, 16, 128, 0)
+    assert lib.qlin_quantize_act_nvfp4(16, 128, 0, 16, ctypes.byref(dk), 16, 256, None) == 1
+    assert lib.qlin_quantize_act_nvfp4_noalloc(16, 0, 256, ctypes.byref(d0), None) == 1
+    f0 = qlin.FP8Desc(16, 16, 0, 256, 0)
+    assert lib.qlin_quantize_act_fp8(16, 0, 256, 16, ctypes.byref(f0), 16, 256, None) == 1
+    assert lib.qlin_quantize_weight(16, 0, 256, 1, ctypes.byref(d0), 16, 256, None) == 1
+    w = qlin.NVFP4Desc(16, 16, 16, 256, 256)
+    assert lib.qlin_gemm_nvfp4(ctypes.byref(d0), ctypes.byref(w), 16, None) == 1
+    a = qlin.NVFP4Desc(16, 16, 16, 128, 256)
+    assert lib.qlin_gemm_nvfp4(ctypes.byref(a), ctypes.byref(d0), 16, None) == 1
+    fw = qlin.FP8Desc(16, 16, 256, 256, 1)
+    assert lib.qlin_gemm_fp8(ctypes.byref(f0), ctypes.byref(fw), 16, None) == 1
+    assert lib.qlin_gemm_bf16(16, 128, 16, 0, 128, 128, 16, None) == 1
+    assert lib.qlin_gemm_fp16(16, 128, 16, 128, 0, 128, 16, None) == 1
