@@ -632,12 +632,15 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
 
 # ------------------------------------------------------------ CPU oracle ---
 
-def cpu_sample_step(aq_full_scale, x_bits, wq, rows, s_next):
-    """The oracle's restatement of one step on a row sample: quantize the
-    sampled activation rows (with the full tensor's dynamic scale), exact fp64
-    GEMM, bf16 rounding, re-quantization."""
+def cpu_sample_step(aq_full_scale, x_bits, wq, rows, s_next, cols=None):
+    """The oracle's restatement of one step on a sample: quantize the sampled
+    activation rows (with the full tensor's dynamic scale), exact fp64 GEMM
+    against the weight rows of the output columns `cols` (a slice; all by
+    default), bf16 rounding, re-quantization."""
     import oracle
     a = oracle.quant_nvfp4(np.ascontiguousarray(x_bits[rows]), aq_full_scale)
+    if cols is not None:
+        wq = (np.ascontiguousarray(wq[0][cols]), np.ascontiguousarray(wq[1][cols]), wq[2])
     y, _, _ = oracle.gemm_nvfp4(a, wq)
     y16 = oracle.round_bf16_array(y)
     oracle.quant_nvfp4(y16, s_next)
@@ -673,30 +676,56 @@ def cpu_baseline(budget_s: float = 15.0):
                       f"weight rows, bf16 round, re-quantize); {dt:.1f} s"}
 
 
-def run_reference(args, dist: Dist):
-    """The reference arm: the CPU oracle as it stands, each step a bounded row
-    sample of the same workload, on this host's cores (rank 0 only)."""
+def run_reference(args, dist: Dist, budget_s: float = 60.0):
+    """The reference arm: the CPU oracle as it stands, on this host's cores
+    (rank 0 only), each step a bounded sample of the same workload sized so
+    that warm-up and steps together take about budget_s: up to 16 token rows
+    against all output columns, or one row against a window of columns when
+    the step count leaves less than a row per step."""
     if dist.rank != 0:
         return None
     oracle, x_bits, wq, s_dec = cpu_setup()
-    rows_per_step = 16
     rng = np.random.default_rng(1)
+    # step cost = fixed + per_out * outputs, from two probes (the step's
+    # whole pipeline: quantize, GEMM, bf16, re-quantize)
+    def probe(n_rows, n_cols):
+        t = time.perf_counter()
+        cpu_sample_step(s_dec, x_bits, wq, np.arange(n_rows), 0.01, slice(0, n_cols))
+        return time.perf_counter() - t
+    probe(1, 64)
+    small, large = probe(1, 64), probe(2, 2048)
+    per_out = max((large - small) / (2 * 2048 - 64), 1e-9)
+    fixed = max(small - 64 * per_out, 0.0)
+    per_step = budget_s / max(args.steps + args.warmup, 1)
+    outs = max(per_step - fixed, 0.0) / per_out
+    rows_per_step = int(min(16, max(1, outs // N)))
+    cols = int(min(N, max(64, outs // rows_per_step // 64 * 64)))
+
+    def sample():
+        r = np.sort(rng.choice(M, rows_per_step, replace=False))
+        c0 = int(rng.integers(0, (N - cols) // 64 + 1)) * 64
+        return r, slice(c0, c0 + cols)
+
     for _ in range(args.warmup):
-        cpu_sample_step(s_dec, x_bits, wq, np.sort(rng.choice(M, rows_per_step, replace=False)), 0.01)
+        r, c = sample()
+        cpu_sample_step(s_dec, x_bits, wq, r, 0.01, c)
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        cpu_sample_step(s_dec, x_bits, wq, np.sort(rng.choice(M, rows_per_step, replace=False)), 0.01)
+        r, c = sample()
+        cpu_sample_step(s_dec, x_bits, wq, r, 0.01, c)
     dt = time.perf_counter() - t0
-    v = 2 * rows_per_step * N * K * args.steps / dt / 1e12
+    v = 2 * rows_per_step * cols * K * args.steps / dt / 1e12
     return {"impl": "reference", "metric": "NVFP4 quantized-linear throughput (TFLOP/s, 2*M*N*K per step)",
             "value": round(v, 6), "unit": "TFLOP/s", "n_gpus": 0, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(dt / args.steps * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64 (oracle)",
             "data": "synthetic (seeded)", "config": {"workload": WORKLOAD, "M": M, "N": N, "K": K,
-                                                     "sample_rows_per_step": rows_per_step},
+                                                     "sample_rows_per_step": rows_per_step,
+                                                     "sample_cols_per_step": cols},
             "cpu_baseline": {"value": round(v, 6), "unit": "TFLOP/s", "cores": oracle.num_threads(),
                              "kind": "oracle",
-                             "sample": f"{rows_per_step} token rows per step of the {M}-row step"},
+                             "sample": f"{rows_per_step} of {M} token rows x {cols} of {N} output "
+                                       f"columns per step"},
             "e2e": {"value": round(v, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
 
