@@ -203,65 +203,102 @@ def run_ours(args, dist: Dist):
         qlin.qlin_quantize_act_nvfp4(xs[r], None, As[r], wss[r])
         qlin.qlin_linear_fused(As[r], Wq[r], ys[r], next_scale, yqs[r])
 
-    # one graph holds S steps, replayed back to back for the timed region.
-    # Timing events (external event nodes) bracket one GEMM in EV_EVERY: an
-    # event node between two kernels breaks their programmatic launch overlap
-    # (measured: events around every GEMM stretched the step from 87 to
-    # 100 us), so the GEMM's duration is sampled rather than bracketed
-    # everywhere.
+    # Steps run as CUDA graphs: a graph of S steps replayed back to back, and
+    # a graph of the remaining n % S steps, so that exactly --warmup and
+    # --steps steps run.  Timing events (external event nodes) bracket one
+    # GEMM in EV_EVERY: an event node between two kernels breaks their
+    # programmatic launch overlap (measured: events around every GEMM
+    # stretched the step from 87 to 100 us), so the GEMM's duration is
+    # sampled rather than bracketed everywhere.
     S = 4 * R
-    try:
-        evs = [(torch.cuda.Event(enable_timing=True, external=True),
-                torch.cuda.Event(enable_timing=True, external=True))
-               for _ in range(S // EV_EVERY)]
-    except TypeError:
-        evs = None
+    graphs = {}
 
-    def s_steps():
-        for i in range(S):
-            r = i % R
-            timed_gemm = evs is not None and i % EV_EVERY == 0
-            qlin.qlin_quantize_act_nvfp4(xs[r], None, As[r], wss[r])
-            if timed_gemm:
-                evs[i // EV_EVERY][0].record(stream)
-            qlin.qlin_linear_fused(As[r], Wq[r], ys[r], next_scale, yqs[r])
-            if timed_gemm:
-                evs[i // EV_EVERY][1].record(stream)
+    def graph_for(n):
+        if n not in graphs:
+            try:
+                evs = [(torch.cuda.Event(enable_timing=True, external=True),
+                        torch.cuda.Event(enable_timing=True, external=True))
+                       for _ in range((n + EV_EVERY - 1) // EV_EVERY)]
+            except TypeError:
+                evs = []
+
+            def steps_n():
+                for i in range(n):
+                    r = i % R
+                    timed_gemm = bool(evs) and i % EV_EVERY == 0
+                    qlin.qlin_quantize_act_nvfp4(xs[r], None, As[r], wss[r])
+                    if timed_gemm:
+                        evs[i // EV_EVERY][0].record(stream)
+                    qlin.qlin_linear_fused(As[r], Wq[r], ys[r], next_scale, yqs[r])
+                    if timed_gemm:
+                        evs[i // EV_EVERY][1].record(stream)
+            graphs[n] = (graph_of(steps_n, torch, stream), evs)
+        return graphs[n]
+
+    def run_steps(n):
+        """Replay exactly n steps; returns the graphs whose events were recorded."""
+        used = []
+        if n >= S:
+            g, evs = graph_for(S)
+            for _ in range(n // S):
+                g.replay()
+            used.append(evs)
+        if n % S:
+            g, evs = graph_for(n % S)
+            g.replay()
+            used.append(evs)
+        return used
 
     for r in range(R):          # first launches outside capture (attributes)
         step(r)
     torch.cuda.synchronize()
-    g = graph_of(s_steps, torch, stream)
-    replays = max(1, args.steps // S)
-    steps = replays * S
-    warm = max(1, -(-args.warmup // S))
-    for _ in range(warm):
-        g.replay()
+    graph_for(S)
+    if args.steps % S:
+        graph_for(args.steps % S)
+    if args.warmup % S:
+        graph_for(args.warmup % S)
+    steps, warm = args.steps, args.warmup
+    run_steps(warm)
     torch.cuda.synchronize()
 
+    # Clock samples: nvidia-smi polls every 200 ms, from just before the timed
+    # region through a sustained window of the same graph replayed for about
+    # a second right after it (a timed region of a few steps is shorter than
+    # the sampling period).
     dist.barrier()
     torch.cuda.synchronize()
     clocks = Clocks(dist.local_rank)
-    time.sleep(0.25)
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t0.record(stream)
-    for _ in range(replays):
-        g.replay()
+    used = run_steps(steps)
     t1.record(stream)
     t1.synchronize()
-    clk = clocks.stop()
     torch.cuda.synchronize()
     dist.barrier()
     sec = dist.max(t0.elapsed_time(t1) / 1e3)
     per_step = sec / steps
     value = STEP_FLOPS * steps * dist.world / sec / 1e12
-
-    if evs:
-        gemm_s = statistics.mean(a.elapsed_time(b) for a, b in evs) / 1e3
+    gemm_samples = [a.elapsed_time(b) / 1e3 for evs in used for a, b in evs]
+    if gemm_samples:
+        gemm_s = statistics.mean(gemm_samples)
     else:
         gemm_s = timed(lambda: qlin.qlin_linear_fused(As[0], Wq[0], ys[0], next_scale, yqs[0]),
                        200, torch, stream)
     gemm_tflops = STEP_FLOPS / gemm_s / 1e12
+    sus_steps = S * max(1, int(1.0 / max(per_step, 1e-6)) // S)
+    s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s0.record(stream)
+    sus_used = run_steps(sus_steps)
+    s1.record(stream)
+    s1.synchronize()
+    clk = clocks.stop()
+    clk["window"] = (f"timed region ({sec * 1e3:.2f} ms) plus a sustained replay of the same "
+                     f"step graph right after it ({sus_steps} steps)")
+    sus_sec = s0.elapsed_time(s1) / 1e3
+    sus_gemm = [a.elapsed_time(b) / 1e3 for evs in sus_used for a, b in evs]
+    sustained = {"steps": sus_steps, "ms_per_step": round(sus_sec / sus_steps * 1e3, 5),
+                 "value": round(STEP_FLOPS * sus_steps / sus_sec / 1e12, 2),
+                 "gemm_us": round(statistics.mean(sus_gemm) * 1e6, 2) if sus_gemm else None}
 
     # ---- end to end through the public API with host buffers: every step
     # copies its x in from pinned host memory and its y out to pinned host
@@ -318,38 +355,59 @@ def run_ours(args, dist: Dist):
            "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2,
            "ms_per_step": round(e2e_sec * 1e3, 4),
            "copies": "pinned host buffers; input copy, compute and output copy on three "
-                     "streams, consecutive steps overlapped"}
+                     "streams, consecutive steps overlapped; y (bf16) is read back every step, "
+                     "the re-quantized y_q stays on the device as the next layer's input"}
+
+    # ---- measured tensor-core ceilings (MMA-only probe, every SM at once)
+    from paper_2609_21849_gb300 import probe
+    ceil = probe.ceilings(sm_max_mhz=float(clk.get("sm_max_mhz") or 2070.0))
+    sms = ceil["nvfp4_pair_256x256x64"]["sms"]
+    mhz = float(clk.get("sm_mhz") or clk.get("sm_max_mhz") or 2070.0)
+    fp4_ceil = ceil["nvfp4_pair_256x256x64"]["flop_per_cycle_per_sm"] * sms * mhz * 1e6 / 1e12
+    fp8_ceil = ceil["fp8_pair_256x256x32"]["flop_per_cycle_per_sm"] * sms * mhz * 1e6 / 1e12
 
     traffic = committed_traffic()
     out = {
         "metric": "NVFP4 quantized-linear throughput (TFLOP/s, 2*M*N*K per step)",
         "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": dist.world, "steps": steps,
-        "warmup": warm * S, "ms_per_step": round(per_step * 1e3, 5), "higher_is_better": True,
+        "warmup": warm, "ms_per_step": round(per_step * 1e3, 5), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "nvfp4 (e2m1 x e4m3 block scales), fp32 accumulate, bf16 out",
         "data": "synthetic (seeded; shapes of FLUX.2-klein at 1024^2, random weights)",
         "config": {"workload": WORKLOAD, "M": M, "N": N, "K": K,
                    "step": "dynamic NVFP4 act quant (one read of x: grid-wide amax + quant) + NVFP4 GEMM + bf16 out + fused NVFP4 requant",
                    "l2": f"{R} rotating input/output sets of {set_bytes / 2**20:.0f} MiB each (> 129 MiB L2)",
-                   "graph": f"CUDA graph of {S} steps replayed {replays}x",
-                   "gemm_timing": f"CUDA events around 1 GEMM in {EV_EVERY} inside the timed graph",
+                   "graph": f"CUDA graphs of {S} steps (replayed {steps // S}x) and of the "
+                            f"remaining {steps % S} steps",
+                   "gemm_timing": f"CUDA events around 1 GEMM in {EV_EVERY} inside the timed graphs "
+                                  f"({len(gemm_samples)} samples)",
                    "parallelism": f"replicas x{dist.world}"},
         "gpu_launches": 2 * steps,
         "clocks": clk,
+        "sustained": sustained,
         "e2e": e2e,
         "roofline": {"kernel": "gemm_kernel<nvfp4, BN=256, requant>", "bound": "tensor",
                      "achieved": round(gemm_tflops, 1),
                      "peak": round(fp4_peak, 1), "unit": "TFLOP/s",
                      "peak_source": f"{pk['source']} bf16 burst {pk['bf16']} TFLOP/s x nominal FP4:BF16 {FP4_PER_BF16:g}",
                      "frac": round(gemm_tflops / fp4_peak, 4),
+                     "mma_ceiling": round(fp4_ceil, 1),
+                     "frac_of_mma_ceiling": round(gemm_tflops / fp4_ceil, 4),
+                     "mma_ceiling_source": f"measured kind::mxf4nvf4 CTA-pair MMA rate "
+                                           f"({ceil['nvfp4_pair_256x256x64']['flop_per_cycle_per_sm']:.0f} "
+                                           f"FLOP/cycle/SM) x {sms} SMs x {mhz:.0f} MHz (median sampled SM clock)",
                      "traffic": traffic,
                      "algorithmic": f"{STEP_FLOPS / 1e9:.2f} GFLOP per launch; {gemm_s * 1e6:.2f} us avg launch"},
+        "mma_probe": ceil,
     }
+    out.update(measure_headline_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak,
+                                     fp4_ceil, fp8_ceil))
     if not args.no_rows:
         out["rows"] = measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak)
     del xs, As, ys, yqs, Wq
     torch.cuda.empty_cache()
     if dist.rank == 0 and not args.no_cpu:
         out["cpu_baseline"] = cpu_baseline(budget_s=15.0)
+        out["cpu_baseline_configs"] = cpu_baseline_configs()
     return out
 
 
@@ -369,88 +427,104 @@ def committed_traffic():
     return rec.get("dram_bytes_per_launch")
 
 
-def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
-    """Secondary rows, each in a CUDA graph, cold L2 by rotating buffers."""
+def g_time(torch, stream, fn, reps_in_graph, replays=20):
+    """Device time per call of fn, captured reps_in_graph times in one CUDA
+    graph and replayed (events on the launching stream)."""
+    fn()
+    torch.cuda.synchronize()
+    g = graph_of(lambda: [fn() for _ in range(reps_in_graph)], torch, stream)
+    g.replay()
+    return timed(g.replay, replays, torch, stream) / reps_in_graph
+
+
+def measure_headline_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak, fp4_ceil,
+                          fp8_ceil):
+    """The quantizer and GEMM rows the metric names (top-level keys of the
+    line): each in a CUDA graph, cold L2 by rotating buffers larger than L2."""
     hbm = pk["hbm_gbs"]
-    rows = {}
-
-    def g_time(fn, reps_in_graph, replays=20):
-        fn()
-        torch.cuda.synchronize()
-        g = graph_of(lambda: [fn() for _ in range(reps_in_graph)], torch, stream)
-        g.replay()
-        return timed(g.replay, replays, torch, stream) / reps_in_graph
-
-    # quantizers on the 4608 x 3072 activations: 8 rotating inputs (226 MB)
-    x_bits = synthetic.act_entry_outliers(2, M, K)
-    R = 8
-    xs = [to_dev(x_bits, torch) for _ in range(R)]
-    qs = [qlin.alloc_nvfp4(M, K) for _ in range(R)]
-    f8 = [qlin.alloc_fp8(M, K, False) for _ in range(R)]
-    wsp = [qlin.alloc_workspace() for _ in range(R)]
+    out = {}
     sc = torch.tensor([np.float32(0.01)], device="cuda")
     c = [0]
 
-    def nxt():
+    def nxt(R):
         c[0] = (c[0] + 1) % R
         return c[0]
-    elems = M * K
-    t = g_time(lambda: (lambda r: qlin.qlin_quantize_act_nvfp4(xs[r], sc, qs[r]))(nxt()), R)
-    rows["a2_quant_nvfp4_static"] = {"us": round(t * 1e6, 2), "GB/s": round(2.5625 * elems / t / 1e9, 1),
-                                     "frac_hbm": round(2.5625 * elems / t / 1e9 / hbm, 3),
-                                     "bytes_per_elem": 2.5625}
-    t = g_time(lambda: (lambda r: qlin.qlin_quantize_act_nvfp4(xs[r], None, qs[r], wsp[r]))(nxt()), R)
-    rows["a1a2_quant_nvfp4_dynamic"] = {"us": round(t * 1e6, 2), "GB/s": round(4.5625 * elems / t / 1e9, 1),
-                                        "frac_hbm": round(4.5625 * elems / t / 1e9 / hbm, 3),
-                                        "bytes_per_elem": 4.5625}
-    t = g_time(lambda: (lambda r: qlin.qlin_quantize_act_fp8(xs[r], sc, f8[r]))(nxt()), R)
-    rows["a3_quant_fp8_static"] = {"us": round(t * 1e6, 2), "GB/s": round(3 * elems / t / 1e9, 1),
-                                   "frac_hbm": round(3 * elems / t / 1e9 / hbm, 3), "bytes_per_elem": 3}
-    t = g_time(lambda: (lambda r: qlin.qlin_quantize_act_fp8(xs[r], None, f8[r], wsp[r]))(nxt()), R)
-    rows["a3_quant_fp8_dynamic"] = {"us": round(t * 1e6, 2), "GB/s": round(5 * elems / t / 1e9, 1),
-                                    "bytes_per_elem": 5}
-    del xs, qs, f8
 
-    # weight quantization (offline): NVFP4 [12288, 3072], FP8 per channel [3072, 3072]
-    (wb,) = synthetic.weights(2, [(N, K)], 0.02)
-    wd = [to_dev(wb, torch) for _ in range(2)]
-    wq = [qlin.alloc_nvfp4(N, K) for _ in range(2)]
-    t = g_time(lambda: (lambda r: qlin.qlin_quantize_weight(wd[r % 2], qlin.QLIN_FMT_NVFP4, wq[r % 2], wsp[r]))(nxt()), 2)
-    rows["a4_weight_quant_nvfp4"] = {"us": round(t * 1e6, 2), "GB/s": round(4.5625 * N * K / t / 1e9, 1)}
-    del wd, wq
+    # ---- NVFP4 / FP8 activation quantizers: x [4608, 3072] (config 3's
+    # activations) and [18432, 3072] (the stack input at B = 4, 113 MB: the
+    # steady-state bandwidth check)
+    quant = {"kernel": "quant_nvfp4_kernel<static> (and onepass / two-pass dynamic routes)",
+             "peak_GB/s": hbm, "peak_source": f"{pk['source']} HBM copy bandwidth"}
+    for (Mq, tag) in ((M, "4608x3072"), (4 * M, "18432x3072")):
+        x_bits = synthetic.act_entry_outliers(2, Mq, K)
+        R = max(2, -(-2 * L2_BYTES // (Mq * K * 2)))        # rotation > 2x L2
+        xs = [to_dev(x_bits, torch) for _ in range(R)]
+        qs = [qlin.alloc_nvfp4(Mq, K) for _ in range(R)]
+        f8 = [qlin.alloc_fp8(Mq, K, False) for _ in range(R)]
+        wsp = [qlin.alloc_workspace() for _ in range(R)]
+        elems = Mq * K
+        row = {"rotating_inputs": R}
+        t = g_time(torch, stream, lambda: (lambda r: qlin.qlin_quantize_act_nvfp4(xs[r], sc, qs[r]))(nxt(R)), R)
+        row["nvfp4_static"] = {"us": round(t * 1e6, 2), "GB/s": round(2.5625 * elems / t / 1e9, 1),
+                               "frac_hbm": round(2.5625 * elems / t / 1e9 / hbm, 3),
+                               "bytes_per_elem": 2.5625}
+        t = g_time(torch, stream, lambda: (lambda r: qlin.qlin_quantize_act_nvfp4(xs[r], None, qs[r], wsp[r]))(nxt(R)), R)
+        row["nvfp4_dynamic"] = {
+            "us": round(t * 1e6, 2),
+            "route": "one read of x (x held on chip)" if Mq * K * 2 <= 152 * 224 * 1024 else "amax pass + quantizer",
+            "GB/s_moved": round((2.5625 if Mq * K * 2 <= 152 * 224 * 1024 else 4.5625) * elems / t / 1e9, 1),
+            "GB/s_at_4.5625": round(4.5625 * elems / t / 1e9, 1),
+            "frac_hbm_moved": round((2.5625 if Mq * K * 2 <= 152 * 224 * 1024 else 4.5625) * elems / t / 1e9 / hbm, 3)}
+        t = g_time(torch, stream, lambda: (lambda r: qlin.qlin_quantize_act_fp8(xs[r], sc, f8[r]))(nxt(R)), R)
+        row["fp8_static"] = {"us": round(t * 1e6, 2), "GB/s": round(3 * elems / t / 1e9, 1),
+                             "frac_hbm": round(3 * elems / t / 1e9 / hbm, 3), "bytes_per_elem": 3}
+        quant[tag] = row
+        del xs, qs, f8, wsp
+        torch.cuda.empty_cache()
+    out["quantizer"] = quant
+    out["quant_nvfp4_static_GBps"] = quant["4608x3072"]["nvfp4_static"]["GB/s"]
+    out["quant_nvfp4_static_frac_hbm"] = quant["4608x3072"]["nvfp4_static"]["frac_hbm"]
+    out["quant_nvfp4_static_frac_hbm_18432x3072"] = quant["18432x3072"]["nvfp4_static"]["frac_hbm"]
 
-    # FP8 linear 4608 x 3072 x 3072 (per-tensor act scale, per-channel W scale)
+    # ---- FP8 linear 4608 x 3072 x 3072 (per-tensor act scale, per-channel W scale)
     x8, w8 = synthetic.fp8_linear()
     Rg = 4
     A8 = [qlin.qlin_quantize_act_fp8(to_dev(x8, torch)) for _ in range(Rg)]
     W8 = [qlin.qlin_quantize_weight(to_dev(w8, torch), qlin.QLIN_FMT_FP8) for _ in range(Rg)]
     y8 = [torch.empty((M, K), dtype=torch.bfloat16, device="cuda") for _ in range(Rg)]
-    t = g_time(lambda: (lambda r: qlin.qlin_gemm_fp8(A8[r % Rg], W8[r % Rg], y8[r % Rg]))(nxt()), Rg * 2)
+    t = g_time(torch, stream, lambda: (lambda r: qlin.qlin_gemm_fp8(A8[r % Rg], W8[r % Rg], y8[r % Rg]))(nxt(Rg)), Rg * 2)
     fl = 2 * M * K * K
-    rows["a6_gemm_fp8"] = {"us": round(t * 1e6, 2), "TFLOP/s": round(fl / t / 1e12, 1),
-                           "frac_fp8_peak": round(fl / t / 1e12 / fp8_peak, 3),
-                           "peak": round(fp8_peak, 1)}
+    out["fp8_gemm"] = {"workload": "4608x3072x3072", "us": round(t * 1e6, 2),
+                       "TFLOP/s": round(fl / t / 1e12, 1),
+                       "frac": round(fl / t / 1e12 / fp8_peak, 3), "peak": round(fp8_peak, 1),
+                       "peak_source": f"{pk['source']} bf16 burst x nominal FP8:BF16 {FP8_PER_BF16:g}",
+                       "frac_of_mma_ceiling": round(fl / t / 1e12 / fp8_ceil, 3),
+                       "mma_ceiling": round(fp8_ceil, 1)}
     del A8, W8, y8
 
-    # NVFP4 GEMM alone (no requant) on the MLP up-projection
+    # ---- NVFP4 GEMM alone (no re-quantization) on the MLP up-projection
     xb, wb2 = synthetic.nvfp4_mlp_up()
     A4 = [qlin.qlin_quantize_act_nvfp4(to_dev(xb, torch)) for _ in range(2)]
     W4 = [qlin.qlin_quantize_weight(to_dev(wb2, torch), qlin.QLIN_FMT_NVFP4) for _ in range(2)]
     y4 = [torch.empty((M, N), dtype=torch.bfloat16, device="cuda") for _ in range(2)]
-    t = g_time(lambda: (lambda r: qlin.qlin_gemm_nvfp4(A4[r % 2], W4[r % 2], y4[r % 2]))(nxt()), 4)
-    rows["a5_gemm_nvfp4"] = {"us": round(t * 1e6, 2), "TFLOP/s": round(STEP_FLOPS / t / 1e12, 1),
-                             "frac_fp4_peak": round(STEP_FLOPS / t / 1e12 / fp4_peak, 3)}
+    t = g_time(torch, stream, lambda: (lambda r: qlin.qlin_gemm_nvfp4(A4[r % 2], W4[r % 2], y4[r % 2]))(nxt(2)), 4)
+    out["nvfp4_gemm"] = {"workload": "4608x12288x3072, bf16 out, no re-quantization",
+                         "us": round(t * 1e6, 2), "TFLOP/s": round(STEP_FLOPS / t / 1e12, 1),
+                         "frac": round(STEP_FLOPS / t / 1e12 / fp4_peak, 3),
+                         "frac_of_mma_ceiling": round(STEP_FLOPS / t / 1e12 / fp4_ceil, 3)}
     # the same linear with the next layer's input quantized at y's own dynamic
     # scale (epilogue amax + a quantizer pass over y: 113 MB read, 35 MB written)
     yq4 = [qlin.alloc_nvfp4(M, N) for _ in range(2)]
     wsd = [qlin.alloc_workspace() for _ in range(2)]
-    t = g_time(lambda: (lambda r: qlin.qlin_linear_dynamic(A4[r % 2], W4[r % 2], y4[r % 2], yq4[r % 2],
-                                                           wsd[r % 2]))(nxt()), 4)
-    rows["f1_linear_dynamic_nvfp4"] = {"us": round(t * 1e6, 2), "TFLOP/s": round(STEP_FLOPS / t / 1e12, 1),
-                                       "note": "GEMM with output-amax epilogue + NVFP4 quantizer over y"}
+    t = g_time(torch, stream, lambda: (lambda r: qlin.qlin_linear_dynamic(A4[r % 2], W4[r % 2], y4[r % 2], yq4[r % 2],
+                                                                          wsd[r % 2]))(nxt(2)), 4)
+    out["f1_linear_dynamic_nvfp4"] = {"us": round(t * 1e6, 2), "TFLOP/s": round(STEP_FLOPS / t / 1e12, 1),
+                                      "vs_plain_gemm": round(t * 1e6 / out["nvfp4_gemm"]["us"], 3),
+                                      "note": "GEMM with output-amax epilogue + NVFP4 quantizer over y"}
     del A4, W4, y4, yq4
 
-    # small-M translator linears (batch 1, 512 tokens), both formats, latency
+    # ---- small-M translator linears (batch 1, 512 tokens), both formats,
+    # against max(compute bound, bytes bound)
     x1, x2, w1, w2 = synthetic.translator()
     res = {}
     for fmt in ("nvfp4", "fp8"):
@@ -459,15 +533,32 @@ def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
                 A = qlin.qlin_quantize_act_nvfp4(to_dev(xb_, torch))
                 W = qlin.qlin_quantize_weight(to_dev(wb_, torch), qlin.QLIN_FMT_NVFP4)
                 fn = lambda A=A, W=W: qlin.qlin_gemm_nvfp4(A, W, yy)
+                nbytes = (A.codes.numel() + A.scales.numel() + W.codes.numel() + W.scales.numel())
+                peak = fp4_peak
             else:
                 A = qlin.qlin_quantize_act_fp8(to_dev(xb_, torch))
                 W = qlin.qlin_quantize_weight(to_dev(wb_, torch), qlin.QLIN_FMT_FP8)
                 fn = lambda A=A, W=W: qlin.qlin_gemm_fp8(A, W, yy)
+                nbytes = A.codes.numel() + W.codes.numel() + 4 * W.rows
+                peak = fp8_peak
             yy = torch.empty((A.rows, W.rows), dtype=torch.bfloat16, device="cuda")
-            t = g_time(fn, 20)
+            nbytes += yy.numel() * 2
+            t = g_time(torch, stream, fn, 20)
             fl = 2 * A.rows * W.rows * A.K
-            res[f"{fmt}_{tag}"] = {"us": round(t * 1e6, 2), "TFLOP/s": round(fl / t / 1e12, 1)}
-    rows["a8_small_m"] = res
+            bound = max(fl / (peak * 1e12), nbytes / (hbm * 1e9))
+            res[f"{fmt}_{tag}"] = {"us": round(t * 1e6, 2), "TFLOP/s": round(fl / t / 1e12, 1),
+                                   "bound_us": round(bound * 1e6, 3),
+                                   "frac_of_bound": round(bound / t, 3),
+                                   "bound": "bytes" if nbytes / (hbm * 1e9) > fl / (peak * 1e12) else "compute"}
+    out["a8_small_m"] = res
+    return out
+
+
+def measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak):
+    """Secondary rows (stack, precision ladder, weight streaming), each in a
+    CUDA graph."""
+    rows = {}
+    wsp = [qlin.alloc_workspace()]
 
     # the 8-block linear stack, B = 1, 2, 4 (one forward = one graph)
     from paper_2609_21849_gb300 import stack
@@ -674,6 +765,129 @@ def cpu_baseline(budget_s: float = 15.0):
             "cores": oracle.num_threads(), "kind": "oracle",
             "sample": f"{n} of {M} token rows of the step (quantize rows, fp64 GEMM vs all 12288 "
                       f"weight rows, bf16 round, re-quantize); {dt:.1f} s"}
+
+
+def _time_rows(step, total_rows, flops_per_row, budget_s, probe_rows):
+    """Time the oracle's step on a row sample of about budget_s (all rows
+    when that fits): the sample grows 2x to 4x per probe until one takes
+    half the budget (at least two probes).  A step costs a fixed part (decoding the weights) plus
+    a part per row; the last two probes give both, and so the full-size time
+    when the sample is not all rows."""
+    def run(n):
+        t0 = time.perf_counter()
+        step(n)
+        return time.perf_counter() - t0
+    pts = []
+    n = min(probe_rows, total_rows)
+    while True:
+        pts.append((n, run(n)))
+        t = pts[-1][1]
+        if n >= total_rows or (t >= budget_s / 2 and len(pts) > 1):
+            break
+        n = min(total_rows, max(2 * n, min(4 * n, int(n * budget_s / max(t, 1e-6)))))
+    n, dt = pts[-1]
+    if len(pts) > 1 and n > pts[-2][0]:
+        per_row = max((dt - pts[-2][1]) / (n - pts[-2][0]), 1e-12)
+        fixed = max(dt - n * per_row, 0.0)
+    else:
+        per_row, fixed = dt / n, 0.0
+    full = dt if n >= total_rows else fixed + per_row * total_rows
+    return {"value": round(flops_per_row * n / dt / 1e12, 6), "unit": "TFLOP/s",
+            "rows": n, "of_rows": total_rows, "seconds": round(dt, 2),
+            "fixed_seconds": round(fixed, 3), "full_size_seconds": round(full, 2),
+            "extrapolated": n < total_rows}
+
+
+def cpu_baseline_configs(budget_s: float = 2.0):
+    """The oracle as it stands, timed on the host cores, single-threaded and
+    on every core, for each workload: the tiny NVFP4 linear, the FP8 linear
+    and the translator linears in full where the budget allows, the MLP
+    up-projection, and the 8-block stack per layer on sampled token rows
+    (extrapolated to all rows, and labelled so).  A step is what the GPU path
+    does: activation quantization with the full tensor's scale, the exact
+    fp64 GEMM, bf16 rounding (and, where the workload has it, the
+    re-quantization of the output); weight quantization is offline."""
+    import oracle
+    from paper_2609_21849_gb300 import synthetic
+    oracle.build()
+    rng = np.random.default_rng(7)
+    cases = {}
+
+    def nvfp4_linear(x, wq, s_next=None):
+        s = oracle.nvfp4_tensor_scale(oracle.amax_bf16(x))
+
+        def step(n):
+            rows = np.sort(rng.choice(x.shape[0], n, replace=False))
+            a = oracle.quant_nvfp4(np.ascontiguousarray(x[rows]), s)
+            y, _, _ = oracle.gemm_nvfp4(a, wq)
+            y16 = oracle.round_bf16_array(y)
+            if s_next is not None:
+                oracle.quant_nvfp4(y16, s_next)
+        return step
+
+    x, w = synthetic.tiny_nvfp4()
+    cases["tiny_nvfp4_128x256x256"] = (nvfp4_linear(x, oracle.quant_nvfp4(w)), 128, 2 * 256 * 256, 16)
+    x8, w8 = synthetic.fp8_linear()
+    wq8 = oracle.quant_fp8_rows(w8)
+    s8 = oracle.fp8_tensor_scale(oracle.amax_bf16(x8))
+
+    def fp8_step(n):
+        rows = np.sort(rng.choice(M, n, replace=False))
+        a = oracle.quant_fp8(np.ascontiguousarray(x8[rows]), s8)
+        y, _, _ = oracle.gemm_fp8(a, wq8)
+        oracle.round_bf16_array(y)
+    cases["fp8_linear_4608x3072x3072"] = (fp8_step, M, 2 * K * K, 4)
+    xu, wu = synthetic.nvfp4_mlp_up()
+    cases["nvfp4_mlp_up_4608x12288x3072_fused"] = (nvfp4_linear(xu, oracle.quant_nvfp4(wu), 0.01),
+                                                   M, 2 * N * K, 4)
+    x1, x2, w1, w2 = synthetic.translator()
+    tq = [(x1, oracle.quant_nvfp4(w1), oracle.quant_fp8_rows(w1)),
+          (x2, oracle.quant_nvfp4(w2), oracle.quant_fp8_rows(w2))]
+
+    def translator_step(n):
+        for xt, wq4, wqf in tq:
+            nvfp4_linear(xt, wq4)(n)
+            sf = oracle.fp8_tensor_scale(oracle.amax_bf16(xt))
+            rows = np.sort(rng.choice(xt.shape[0], n, replace=False))
+            y, _, _ = oracle.gemm_fp8(oracle.quant_fp8(np.ascontiguousarray(xt[rows]), sf), wqf)
+            oracle.round_bf16_array(y)
+    cases["translator_512x2560x1024_512x1024x2560_nvfp4_fp8"] = (
+        translator_step, 512, 2 * 2 * (2560 * 1024 + 1024 * 2560), 4)
+
+    # the stack: one block's 4 layers chained on the sampled rows (layers are
+    # row-local once their static scales are fixed; the 8 blocks have the
+    # same shapes, so the stack takes 8x a block)
+    wl = list(synthetic.stack_weights(1, 4))
+    wsq = [(name, oracle.quant_nvfp4(wb)) for (_, name, wb) in wl]
+    del wl
+    xs5 = synthetic.stack_input(1)
+    s5 = oracle.nvfp4_tensor_scale(oracle.amax_bf16(xs5))
+
+    def stack_step(n):
+        rows = np.sort(rng.choice(xs5.shape[0], n, replace=False))
+        a = oracle.quant_nvfp4(np.ascontiguousarray(xs5[rows]), s5)
+        for name, wq in wsq:
+            y, _, _ = oracle.gemm_nvfp4(a, wq)
+            y16 = oracle.round_bf16_array(y)
+            win = np.ascontiguousarray(y16[:, 2 * K:] if name == "qkv" else y16)
+            a = oracle.quant_nvfp4(win, oracle.nvfp4_tensor_scale(oracle.amax_bf16(win)))
+    per_row5 = 2 * (3 * K * K + K * K + 2 * N * K)
+
+    res = {}
+    all_threads = oracle.num_threads()
+    for threads in (1, all_threads):
+        oracle.set_num_threads(threads)
+        tag = "1_thread" if threads == 1 else f"{threads}_threads"
+        for name, (fn, total, fpr, probe_n) in cases.items():
+            res.setdefault(name, {})[tag] = _time_rows(fn, total, fpr, budget_s, probe_n)
+        r5 = _time_rows(stack_step, M, per_row5, budget_s, 1)
+        r5["stack_full_size_seconds"] = {f"B{b}": round(8 * b * r5["full_size_seconds"], 1)
+                                         for b in (1, 2, 4)}
+        r5["note"] = ("one block's 4 layers chained on sampled token rows; the 8-block stack "
+                      "at 4608*B rows extrapolated as 8 blocks x B x (fixed + per-row cost)")
+        res.setdefault("stack_block", {})[tag] = r5
+    oracle.set_num_threads(all_threads)
+    return {"kind": "oracle", "cores": all_threads, "configs": res}
 
 
 def run_reference(args, dist: Dist, budget_s: float = 60.0):

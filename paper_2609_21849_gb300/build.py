@@ -16,6 +16,9 @@ INCLUDE = os.path.join(ROOT, "include")
 LIB_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(LIB_DIR, "libqlin.so")
 SOURCES = ["qlin_api.cu", "qlin_quant.cu", "qlin_gemm.cu"]
+# the tensor-core rate probe of the measurement harness: a library of its own
+PROBE_LIB = os.path.join(LIB_DIR, "libqlin_probe.so")
+PROBE_SOURCES = ["qlin_probe.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -33,18 +36,24 @@ def _flags():
 
 def _inputs():
     deps = [os.path.join(CSRC, f) for f in os.listdir(CSRC)]
-    deps.append(os.path.join(INCLUDE, "qlin.h"))
+    deps += [os.path.join(INCLUDE, f) for f in os.listdir(INCLUDE)]
     return deps
 
 
+def _fresh(lib):
+    if not os.path.exists(lib):
+        return False
+    t = os.path.getmtime(lib)
+    return all(os.path.getmtime(d) <= t for d in _inputs())
+
+
 def build(force: bool = False, verbose: bool = False) -> str:
+    """Build libqlin.so and libqlin_probe.so (all translation units compiled
+    in parallel); returns the path of libqlin.so."""
     os.makedirs(LIB_DIR, exist_ok=True)
-    if not force and os.path.exists(LIB):
-        t = os.path.getmtime(LIB)
-        if all(os.path.getmtime(d) <= t for d in _inputs()):
-            return LIB
+    if not force and _fresh(LIB) and _fresh(PROBE_LIB):
+        return LIB
     cc = nvcc()
-    objs = []
 
     def compile_one(src):
         obj = os.path.join(LIB_DIR, src.replace(".cu", ".o"))
@@ -56,14 +65,17 @@ def build(force: bool = False, verbose: bool = False) -> str:
             sys.stderr.write(r.stdout + r.stderr)
         return obj
 
-    with cf.ThreadPoolExecutor(len(SOURCES)) as ex:
-        objs = list(ex.map(compile_one, SOURCES))
-    tmp = LIB + ".tmp"
-    cmd = [cc] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs + ["-ldl", "-lpthread", "-lrt"]
-    r = subprocess.run(cmd, capture_output=True, text=True)
-    if r.returncode != 0:
-        raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
+    srcs = SOURCES + PROBE_SOURCES
+    with cf.ThreadPoolExecutor(len(srcs)) as ex:
+        objs = dict(zip(srcs, ex.map(compile_one, srcs)))
+    for lib, group in ((LIB, SOURCES), (PROBE_LIB, PROBE_SOURCES)):
+        tmp = lib + ".tmp"
+        cmd = ([cc] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + [objs[f] for f in group]
+               + ["-ldl", "-lpthread", "-lrt"])
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
+        os.replace(tmp, lib)
     return LIB
 
 

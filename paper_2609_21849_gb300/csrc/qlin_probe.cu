@@ -1,0 +1,206 @@
+// Tensor-core rate probe (measurement only, not part of the linear layer):
+// back-to-back tcgen05.mma instructions of one kind and shape from one thread
+// per CTA (or CTA pair), on every SM at once, operands resident in shared
+// memory.  It gives the MMA ceiling that the GEMMs' roofline fractions are
+// also reported against, in FLOP per SM cycle (clock-independent) and in
+// FLOP/s at the clock the probe ran at.
+//
+// Only the instruction forms the GEMMs issue are used: kind::mxf4nvf4
+// block_scale scale_vec::4X (NVFP4), kind::f8f6f4 (E4M3) and kind::f16
+// (bf16), each as cta_group::1 (M = 128) and cta_group::2 (M = 256).
+#include <cstdio>
+
+#include "qlin_device.cuh"
+#include "qlin_probe.h"
+
+namespace qlin {
+namespace {
+
+constexpr int kProbeThreads = 128;
+constexpr int kASmem = 128 * 128;       // 128 rows x 128 bytes of K
+constexpr int kBSmemMax = 256 * 128;    // up to 256 rows x 128 bytes
+constexpr int kSfSmem = 4096;           // scale atoms (NVFP4)
+// Requested shared memory: more than half an SM's, so that no SM holds two
+// probe CTAs (each allocates all 512 TMEM columns; two CTA pairs sharing SMs
+// could otherwise wait on each other's allocations).
+constexpr int kProbeSmem = 160 * 1024;
+static_assert(1024 + kASmem + kBSmemMax + kSfSmem <= kProbeSmem, "probe buffers");
+
+__device__ __forceinline__ uint32_t hash32(uint32_t x) {
+  x ^= x >> 16;
+  x *= 0x7FEB352Du;
+  x ^= x >> 15;
+  x *= 0x846CA68Bu;
+  x ^= x >> 16;
+  return x;
+}
+
+// Bounded wait on an mbarrier phase (iteration limit of a few seconds at the
+// try_wait suspend hint; records an error flag).
+__device__ __forceinline__ bool probe_wait(uint64_t* bar, uint32_t parity, unsigned* err) {
+  for (uint32_t i = 0; i < (1u << 17); ++i)
+    if (mbar_try_wait(smem_u32(bar), parity)) return true;
+  atomicExch(err, kErrTimeout);
+  return false;
+}
+
+// kKind: 4 = NVFP4 (mxf4nvf4, K = 64), 8 = FP8 (f8f6f4, K = 32), 16 = bf16
+// (f16, K = 16); every instruction reads 32 bytes of K per operand row.
+template <int kKind, bool kPair, int kN>
+__global__ void __launch_bounds__(kProbeThreads, 1)
+    mma_probe_kernel(int iters, unsigned long long* out, unsigned* err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = base;
+  uint8_t* sB = base + kASmem;
+  uint8_t* sSF = sB + kBSmemMax;
+  __shared__ uint64_t bar;
+  __shared__ uint32_t tmem_slot;
+  // operands: hashed bytes (typical bit toggling), finite in every format
+  // (bf16 / E4M3 exponent fields kept below all-ones); scales 1.0 (0x38)
+  for (int i = threadIdx.x; i < (kASmem + kBSmemMax) / 4; i += kProbeThreads) {
+    uint32_t v = hash32((uint32_t)i * 2654435761u + blockIdx.x);
+    if (kKind == 8) v &= 0xBFBFBFBFu;          // E4M3: no NaN codes
+    if (kKind == 16) v &= 0xBFFFBFFFu;         // bf16: exponent below all-ones
+    reinterpret_cast<uint32_t*>(base)[i] = v;
+  }
+  for (int i = threadIdx.x; i < kSfSmem / 4; i += kProbeThreads)
+    reinterpret_cast<uint32_t*>(sSF)[i] = 0x38383838u;
+  const uint32_t rank = kPair ? cluster_ctarank() : 0;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    mbar_fence_init();
+  }
+  if ((threadIdx.x >> 5) == 1) {
+    if (kPair)
+      tmem_alloc_pair(&tmem_slot, 512);
+    else
+      tmem_alloc(&tmem_slot, 512);
+  }
+  fence_proxy_async_smem();
+  tc_fence_before();
+  if (kPair)
+    cluster_sync();
+  else
+    __syncthreads();
+  tc_fence_after();
+  const uint32_t tb = tmem_slot;
+  if (threadIdx.x == 0 && rank == 0) {
+    constexpr int kM = kPair ? 256 : 128;
+    const uint32_t idesc = kKind == 4 ? idesc_nvfp4(kN, kM)
+                           : kKind == 8 ? idesc_fp8(kN, kM)
+                                        : idesc_bf16(kN, kM);
+    const uint32_t a = smem_u32(sA), b = smem_u32(sB), sf = smem_u32(sSF);
+    const uint32_t sf_t = tb + 256;   // scale columns: A at +0, B atoms at +4, +8
+    if (kKind == 4) {
+      for (int r = 0; r < 3; ++r) {
+        if (kPair)
+          tc_cp_scales_pair(sf_t + 4 * r, sdesc_scales(sf + 512 * r));
+        else
+          tc_cp_scales(sf_t + 4 * r, sdesc_scales(sf + 512 * r));
+      }
+    }
+    if (kPair)
+      tc_commit_pair_mc(&bar, 1);
+    else
+      tc_commit(&bar);
+    bool ok = probe_wait(&bar, 0, err);
+    tc_fence_after();
+    const unsigned long long c0 = clock64();
+    const uint64_t t0 = global_timer_ns();
+    for (int i = 0; ok && i < iters; ++i) {
+      const uint32_t j = (uint32_t)(i & 3) * 32;
+      const uint64_t ad = sdesc_k128(a + j), bd = sdesc_k128(b + j);
+      const uint32_t acc = i > 0 ? 1u : 0u;
+      if (kKind == 4) {
+        if (kPair)
+          mma_nvfp4_pair(tb, ad, bd, idesc, sf_t, sf_t + 4, acc);
+        else
+          mma_nvfp4(tb, ad, bd, idesc, sf_t, sf_t + 4, acc);
+      } else if (kKind == 8) {
+        if (kPair)
+          mma_fp8_pair(tb, ad, bd, idesc, acc);
+        else
+          mma_fp8(tb, ad, bd, idesc, acc);
+      } else {
+        if (kPair)
+          mma_bf16_pair(tb, ad, bd, idesc, acc);
+        else
+          mma_bf16(tb, ad, bd, idesc, acc);
+      }
+    }
+    if (kPair)
+      tc_commit_pair_mc(&bar, 1);
+    else
+      tc_commit(&bar);
+    ok = ok && probe_wait(&bar, 1, err);
+    const unsigned long long c1 = clock64();
+    const uint64_t t1 = global_timer_ns();
+    const int slot = (int)blockIdx.x / (kPair ? 2 : 1);
+    out[2 * slot] = ok ? c1 - c0 : 0ull;
+    out[2 * slot + 1] = ok ? t1 - t0 : 0ull;
+  }
+  tc_fence_before();
+  if (kPair)
+    cluster_sync();
+  else
+    __syncthreads();
+  if ((threadIdx.x >> 5) == 1) {
+    tc_fence_after();
+    if (kPair)
+      tmem_dealloc_pair(tb, 512);
+    else
+      tmem_dealloc(tb, 512);
+  }
+}
+
+template <int kKind, bool kPair, int kN>
+cudaError_t launch_probe(int ctas, int iters, unsigned long long* out, unsigned* err,
+                         cudaStream_t s) {
+  auto kern = mma_probe_kernel<kKind, kPair, kN>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       kProbeSmem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg{};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kPair ? 2 : 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3((unsigned)ctas, 1, 1);
+  cfg.blockDim = dim3(kProbeThreads, 1, 1);
+  cfg.dynamicSmemBytes = kProbeSmem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, iters, out, err);
+}
+
+}  // namespace
+}  // namespace qlin
+
+using namespace qlin;
+
+extern "C" int qlin_probe_mma(int kind, int pair, int n, int ctas, int iters,
+                              unsigned long long* out, unsigned* err, void* stream) {
+  if (out == nullptr || err == nullptr || iters < 1 || ctas < 1) return 1;
+  if (pair && ctas % 2 != 0) return 1;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaSuccess;
+  bool matched = false;
+#define QLIN_PROBE_CASE(K, P, N)                                      \
+  if (kind == K && (pair != 0) == P && n == N) {                      \
+    matched = true;                                                   \
+    e = launch_probe<K, P, N>(ctas, iters, out, err, s);              \
+  }
+  QLIN_PROBE_CASE(4, true, 256);
+  QLIN_PROBE_CASE(4, false, 256);
+  QLIN_PROBE_CASE(4, false, 128);
+  QLIN_PROBE_CASE(8, true, 256);
+  QLIN_PROBE_CASE(8, false, 256);
+  QLIN_PROBE_CASE(16, true, 256);
+#undef QLIN_PROBE_CASE
+  if (!matched) return 1;
+  return e == cudaSuccess ? 0 : 4;
+}

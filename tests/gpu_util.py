@@ -75,3 +75,77 @@ def requant_agreement(gpu_codes, gpu_canon, y16_gpu, y16_ref, s_next):
     bad = np.argwhere(same_in & ~same_out)
     assert bad.size == 0, ("re-quantized block differs on identical inputs", bad[:5])
     return same_out.mean()
+
+
+def stratified_rows(M: int, n: int, seed: int = 0) -> np.ndarray:
+    """Rows covering every 128-row M tile, cycling through the four 32-lane
+    quarters of the tile's TMEM accumulator from tile to tile, plus the first
+    and last rows, topped up with random rows to about n (sorted, unique)."""
+    rng = np.random.default_rng(seed)
+    rows = {0, M - 1}
+    for t in range((M + 127) // 128):
+        q = t % 4
+        r = t * 128 + q * 32 + int(rng.integers(0, 32))
+        rows.add(min(r, M - 1))
+    extra = max(0, n - len(rows))
+    if extra:
+        rows |= set(rng.choice(M, size=min(extra, M), replace=False).tolist())
+    return np.array(sorted(rows), np.int64)
+
+
+def assert_requant_exact(gpu_codes, gpu_canon, y16_gpu, s_next, what=""):
+    """The fused re-quantization of a layer's own bf16 output: its codes and
+    scales must equal the oracle's NVFP4 quantization of that same bf16
+    output with the same static tensor scale, bit for bit (every block)."""
+    ref = oracle.quant_nvfp4(np.ascontiguousarray(y16_gpu), s_next)
+    bad = np.argwhere(gpu_canon != ref[1])
+    assert bad.size == 0, (what, "re-quantized scales differ", bad[:5])
+    bad = np.argwhere(gpu_codes != ref[0])
+    assert bad.size == 0, (what, "re-quantized codes differ", bad[:5])
+    return ref
+
+
+def check_stack_layers(st, x_bits, wqs, rows, s0, what=""):
+    """Per-layer oracle parity of a linear stack's forward on the given token
+    rows.  Layer i's input is checked bit-exactly against the oracle's
+    quantization of the previous layer's bf16 output (for the first layer, of
+    the stack input x with tensor scale s0), and its bf16 output is checked
+    within GEMM_TOL against the oracle's exact fp64 product of that input and
+    the oracle-quantized weight wqs[i].  Returns the worst normalised error."""
+    Rt = torch.from_numpy(rows).cuda()
+    a_ref = oracle.quant_nvfp4(np.ascontiguousarray(x_bits[rows]), s0)
+    codes, canon, s = nvfp4_to_host(st.a0)
+    assert s == np.float32(s0), (what, "input tensor scale")
+    assert np.array_equal(codes[rows], a_ref[0]) and np.array_equal(canon[rows], a_ref[1]), \
+        (what, "stack input quantization")
+    worst = 0.0
+    for i, l in enumerate(st.layers):
+        yref, na, nw = oracle.gemm_nvfp4(a_ref, wqs[i])
+        yb = bf16_bits(l.y.index_select(0, Rt))
+        err, exact = gemm_errors(yb, yref, na, nw)
+        assert err.max() <= GEMM_TOL, (what, i, l.block, l.name, err.max())
+        worst = max(worst, float(err.max()))
+        s_next = np.float32(f32(l.next_scale)[0])
+        codes, canon, s = nvfp4_to_host(l.out_q)
+        assert s == s_next, (what, i, "re-quantized tensor scale")
+        win = np.ascontiguousarray(yb[:, l.rq_col0:l.rq_col0 + l.rq_cols])
+        a_ref = assert_requant_exact(codes[rows], canon[rows], win, s_next, (what, i))
+    return worst
+
+
+def oracle_stack_scales(x_bits, wlist, wqs, rows, v_col0):
+    """Static next-layer scales of a linear stack, calibrated by the oracle:
+    its own chain on the given token rows (exact GEMM, bf16 rounding, dynamic
+    tensor scale of each re-quantized window), as post-training calibration
+    does.  Returns (input tensor scale s0, per-layer next scales)."""
+    s0 = oracle.nvfp4_tensor_scale(oracle.amax_bf16(x_bits))
+    a = oracle.quant_nvfp4(np.ascontiguousarray(x_bits[rows]), s0)
+    scales = []
+    for (_, name, _), wq in zip(wlist, wqs):
+        yref, _, _ = oracle.gemm_nvfp4(a, wq)
+        c0 = v_col0 if name == "qkv" else 0
+        win = np.ascontiguousarray(oracle.round_bf16_array(yref)[:, c0:])
+        s_next = oracle.nvfp4_tensor_scale(oracle.amax_bf16(win))
+        scales.append(s_next)
+        a = oracle.quant_nvfp4(win, s_next)
+    return s0, scales

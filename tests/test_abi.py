@@ -16,8 +16,8 @@ def lib():
     return qlin.load_library()
 
 
-def _declared():
-    src = open(os.path.join(ROOT, "include", "qlin.h")).read()
+def _declared(header="qlin.h"):
+    src = open(os.path.join(ROOT, "include", header)).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
     return sorted(set(re.findall(r"\b(qlin_\w+)\s*\(", src)))
 
@@ -34,6 +34,24 @@ def test_every_declared_symbol_is_exported(lib):
     for name in _declared():
         assert hasattr(lib, name), name
     assert sorted(qlin.EXPORTS) == _declared()
+
+
+def test_probe_library_exports_its_header(lib):
+    # the tensor-core rate probe of the measurement harness: its own library
+    from paper_2609_21849_gb300 import build
+    probe = ctypes.CDLL(build.PROBE_LIB)
+    names = _declared("qlin_probe.h")
+    assert names == ["qlin_probe_mma"]
+    for name in names:
+        assert hasattr(probe, name), name
+    f = probe.qlin_probe_mma
+    f.restype = ctypes.c_int
+    f.argtypes = [ctypes.c_int] * 5 + [ctypes.c_void_p] * 3
+    one = ctypes.c_ulonglong(0)
+    # argument errors are returned before any launch
+    assert f(4, 1, 256, 3, 16, ctypes.addressof(one), ctypes.addressof(one), None) == 1  # odd pair grid
+    assert f(4, 0, 64, 2, 16, ctypes.addressof(one), ctypes.addressof(one), None) == 1   # no such case
+    assert f(4, 0, 256, 2, 16, None, None, None) == 1
 
 
 def test_scale_bytes_and_workspace(lib):

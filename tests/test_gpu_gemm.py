@@ -1,7 +1,9 @@
 """GPU parity of the block-scaled GEMMs (Sec. 4: the quantized linears run on
 the NVFP4 / FP8 tensor cores).  Operands are quantized on the GPU and checked
 bit-exact against the oracle; the bf16 output is checked against the oracle's
-exact fp64 result with |y - y_exact| / (||a_m|| ||w_n||) <= 2e-3."""
+exact fp64 result with |y - y_exact| / (||a_m|| ||w_n||) <= 2e-3, and at least
+99% of the outputs must equal the correctly rounded bf16 of the exact result
+(the kernels differ from it only by fp32 accumulation order)."""
 import numpy as np
 import pytest
 
@@ -14,7 +16,7 @@ pytestmark = pytest.mark.gpu
 
 if torch.cuda.is_available():
     from gpu_util import (GEMM_TOL, assert_nvfp4_equal, bf16_bits, f32, gemm_errors,
-                          sample_rows, to_dev, u8)
+                          sample_rows, stratified_rows, to_dev, u8)
 
 
 def _check_nvfp4(x, w, rows=None, label=""):
@@ -32,7 +34,7 @@ def _check_nvfp4(x, w, rows=None, label=""):
     err, exact = gemm_errors(yb, yref, na, nw)
     assert np.all(np.isfinite(err)), label
     assert err.max() <= GEMM_TOL, (label, err.max(), np.unravel_index(err.argmax(), err.shape))
-    assert exact >= 0.5, (label, exact)
+    assert exact >= 0.99, (label, exact)
     return err.max(), exact
 
 
@@ -50,7 +52,7 @@ def _check_fp8(x, w, rows=None, label=""):
     err, exact = gemm_errors(bf16_bits(y)[sel], yref, na, nw)
     assert np.all(np.isfinite(err)), label
     assert err.max() <= GEMM_TOL, (label, err.max())
-    assert exact >= 0.5, (label, exact)
+    assert exact >= 0.99, (label, exact)
     return err.max(), exact
 
 
@@ -70,7 +72,7 @@ RAGGED = [(1, 64, 64), (77, 320, 192), (300, 128, 512), (129, 576, 1088),
 def test_nvfp4_ragged(M, N, K):
     x = synthetic.act_entry_outliers(M + N + K, M, K)
     (w,) = synthetic.weights(M + N + K, [(N, K)], 0.02)
-    rows = sample_rows(M, 48, seed=M) if M > 64 else None
+    rows = stratified_rows(M, 48, seed=M) if M > 64 else None
     _check_nvfp4(x, w, rows, f"nvfp4 {M}x{N}x{K}")
 
 
@@ -78,20 +80,22 @@ def test_nvfp4_ragged(M, N, K):
 def test_fp8_ragged(M, N, K):
     x = synthetic.act_channel_gain(M + N + K, M, K)
     (w,) = synthetic.weights(M + N + K, [(N, K)], 0.02)
-    rows = sample_rows(M, 48, seed=M) if M > 64 else None
+    rows = stratified_rows(M, 48, seed=M) if M > 64 else None
     _check_fp8(x, w, rows, f"fp8 {M}x{N}x{K}")
 
 
 def test_nvfp4_mlp_up_full_size():
-    # 4608 x 12288 x 3072, in the launch configuration the benchmark times
+    # 4608 x 12288 x 3072, in the launch configuration the benchmark times;
+    # every output is compared with the oracle (every tile position and TMEM
+    # lane quarter)
     x, w = synthetic.nvfp4_mlp_up()
-    e, ex = _check_nvfp4(x, w, sample_rows(x.shape[0], 40), "mlp-up")
+    e, ex = _check_nvfp4(x, w, None, "mlp-up")
     print(f"mlp-up nvfp4: max err {e:.3e}, exact {ex:.4f}")
 
 
 def test_fp8_linear_full_size():
     x, w = synthetic.fp8_linear()
-    e, ex = _check_fp8(x, w, sample_rows(x.shape[0], 40), "fp8-linear")
+    e, ex = _check_fp8(x, w, None, "fp8-linear")   # every output
     print(f"fp8 linear: max err {e:.3e}, exact {ex:.4f}")
 
 
@@ -158,5 +162,5 @@ def test_nvfp4_ragged_pair_tiles_partial_last_wave():
     M, N, K = 4500, 12224, 1024
     x = synthetic.act_entry_outliers(77, M, K)
     (w,) = synthetic.weights(78, [(N, K)], 0.02)
-    rows = np.unique(np.concatenate([sample_rows(M, 40, seed=5), np.arange(M - 20, M)]))
+    rows = np.unique(np.concatenate([stratified_rows(M, 64, seed=5), np.arange(M - 20, M)]))
     _check_nvfp4(x, w, rows, "pair tiles 4500x12224x1024")

@@ -1,13 +1,19 @@
 """Weight streaming on the GPU (Sec. 4, "Weight streaming"): the streamed
 forward of the linear stack must give outputs bit-identical to the fully
-resident forward, since only where the weights live changes."""
+resident forward, since only where the weights live changes, and each
+streamed layer must match the oracle."""
+import numpy as np
 import pytest
 
 torch = pytest.importorskip("torch")
 
+import oracle
 from paper_2609_21849_gb300 import qlin, stack, streaming, synthetic
 
 pytestmark = pytest.mark.gpu
+
+if torch.cuda.is_available():
+    from gpu_util import check_stack_layers, oracle_stack_scales, stratified_rows, to_dev
 
 
 def _outputs(st):
@@ -72,3 +78,29 @@ def test_streamed_forward_in_cuda_graph():
     torch.cuda.synchronize()
     assert qlin.qlin_sync_status() == 0
     _assert_same(st, ref, "graph")
+
+
+@pytest.mark.parametrize("frac,slots", [(0.25, 2), (0.0, 3)])
+def test_streamed_forward_matches_oracle(frac, slots):
+    # Seeded 2-block stack (the stack's own weight and input recipes), static
+    # scales calibrated by the oracle; after a streamed forward (most layers
+    # copied from pinned host memory into the device slots), every layer is
+    # checked against the oracle on rows covering every 128-row tile.
+    wlist = list(synthetic.stack_weights(2, 4))
+    wqs = [oracle.quant_nvfp4(w) for (_, _, w) in wlist]
+    x = synthetic.stack_input(1)
+    M = x.shape[0]
+    s0, scales = oracle_stack_scales(x, wlist, wqs, stratified_rows(M, 48, seed=3), stack.V_COL0)
+    st = stack.build_stack(1, weights=wlist)
+    st.set_next_scales(scales)
+    ss = streaming.StreamedStack(st, frac, n_slots=slots)
+    s = torch.cuda.Stream()
+    xd = to_dev(x)
+    with torch.cuda.stream(s):
+        ss.forward(xd, s)
+    torch.cuda.synchronize()
+    assert qlin.qlin_sync_status() == 0
+    assert sum(not r for r in ss.resident) >= 6, ss.resident   # most layers streamed
+    worst = check_stack_layers(st, x, wqs, stratified_rows(M, 128, seed=4), s0,
+                               f"streamed {frac} x{slots}")
+    print(f"streamed forward ({frac:.2f} resident, {slots} slots): worst error {worst:.2e}")

@@ -6,7 +6,8 @@ stall on cudaMalloc.  This entry point quantizes with the dynamic tensor scale
 like qlin_quantize_act_nvfp4, but keeps its amax scratch in the library's own
 static device array instead of a caller workspace.  Here it must reproduce the
 workspace entry point's codes, scales and tensor scale exactly, on two calls in
-a row (the second with a smaller amax, so stale scratch would show).
+a row (the second with a smaller amax, so stale scratch would show), and, on an
+input too large for the one-read route, the oracle's.
 
 This file is collected last on purpose; it passes alone in a fresh process and
 after the other tests.
@@ -16,6 +17,7 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
+import oracle
 from paper_2609_21849_gb300 import qlin, synthetic
 
 pytestmark = pytest.mark.gpu
@@ -53,6 +55,22 @@ def test_noalloc_full_size_activation():
     assert qlin.qlin_sync_status() == 0
     _same(a, ref)
     _same(b, ref)
+
+
+def test_noalloc_two_pass_route_matches_oracle_twice():
+    # x [9216, 4096] (75 MB) does not fit in the grid's shared memory, so the
+    # entry point takes its two-pass route (an amax pass into the static
+    # scratch, then the quantizer).  Two calls in a row, the second with a
+    # smaller amax: a stale amax left in the scratch would change its scale.
+    M, K = 9216, 4096
+    for bits in (synthetic.act_entry_outliers(31, M, K), synthetic.act_normal(32, M, K)):
+        out = qlin.qlin_quantize_act_nvfp4_noalloc(_dev(bits), qlin.alloc_nvfp4(M, K))
+        assert qlin.qlin_sync_status() == 0
+        rc, rs, sd = oracle.quant_nvfp4(bits)
+        assert np.float32(out.tensor_scale.item()).view(np.uint32) == np.float32(sd).view(np.uint32)
+        assert np.array_equal(out.codes.cpu().numpy(), rc)
+        canon = oracle.unswizzle_scales(out.scales.cpu().numpy(), M, K)
+        assert np.array_equal(canon, rs)
 
 
 def test_noalloc_rejects_bad_arguments():
