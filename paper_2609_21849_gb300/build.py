@@ -30,8 +30,11 @@ def nvcc() -> str:
 
 
 def _flags():
+    # QLIN_BUILD_DEFINES: extra -D options (the kernels' build-time layout
+    # choices, e.g. "-DQLIN_WIDE_NVFP4=0"); empty for the default build
+    extra = os.environ.get("QLIN_BUILD_DEFINES", "").split()
     return ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
-                   "-I" + INCLUDE, "-I" + CSRC]
+                   "-I" + INCLUDE, "-I" + CSRC] + extra
 
 
 def _inputs():

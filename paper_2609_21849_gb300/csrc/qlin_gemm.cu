@@ -26,9 +26,9 @@
 //               MMA stream, each warp the atoms of half the stage's MMA steps.
 //   warp 4      NVFP4 pair tiles: TMA producer of the scale atoms.
 //   last 8      epilogue: tcgen05.ld of the accumulator, alpha, 16-bit
-//               rounding; NVFP4 tiles store y by TMA through swizzled staging,
-//               FP8 / 16-bit pair tiles store it straight from registers (the
-//               staging's shared memory holds a seventh stage instead);
+//               rounding; pair tiles store y straight from registers (FP8 /
+//               16-bit tiles use the freed staging memory for a seventh
+//               stage), single-CTA tiles by TMA through swizzled staging;
 //               optional re-quantization of the 16-bit values, one row per
 //               thread, and optional output amax.
 // Every wait is bounded (see WaitCtl).
@@ -56,6 +56,17 @@ constexpr int kEpiWarps = 8;
 #endif
 #ifndef QLIN_TMA_SPLIT
 #define QLIN_TMA_SPLIT 1
+#endif
+// NVFP4 pair tiles store y straight from registers (no staging boxes and no
+// TMA stores sharing the copy engine with the operand loads)
+#ifndef QLIN_FP4_DIRECT_STORE
+#define QLIN_FP4_DIRECT_STORE 1
+#endif
+// Tile order: cluster tiles are visited in groups of this many M tile groups
+// (0: all of M, i.e. M fastest within each N tile; on the 4608 x 12288 x 3072
+// NVFP4 GEMM groups of 1 to 9 measured 3-6% slower)
+#ifndef QLIN_GROUP_M
+#define QLIN_GROUP_M 0
 #endif
 constexpr int kSmemBudget = 232448 - 2048;  // opt-in shared memory minus barriers/alignment
 constexpr int kSplit = QLIN_TMA_SPLIT;      // row boxes per operand tile and stage
@@ -86,11 +97,13 @@ struct Cfg {
   static constexpr int kSfaBytes = kFp4 ? kStepsPerStage * 512 : 0;
   static constexpr int kSfbBytes = kFp4 ? kSfbAtoms * kStepsPerStage * 512 : 0;
   static constexpr int kStageBytes = kABytes + kBBytes + kSfaBytes + kSfbBytes;
-  // FP8 / 16-bit pair tiles store y straight from registers (each thread
-  // its row's 64 bytes per 32 columns), which frees the staging boxes for a
-  // seventh pipeline stage; otherwise per epilogue warp two 32 x 32 bf16
-  // boxes (2 KB each) stage TMA stores
-  static constexpr bool kDirectStore = !kFp4 && kPair && kBN == 256;
+  // Pair tiles store y straight from registers (each thread its row's 64
+  // bytes per 32 columns): for FP8 / 16-bit tiles the staging's shared memory
+  // holds a seventh pipeline stage, and for NVFP4 tiles the operand loads
+  // keep the copy engine to themselves (measured 70.1 -> 66.7 us on the
+  // 4608 x 12288 x 3072 GEMM).  Otherwise per epilogue warp two 32 x 32 bf16
+  // boxes (2 KB each) stage TMA stores.
+  static constexpr bool kDirectStore = kPair && kBN == 256 && (!kFp4 || QLIN_FP4_DIRECT_STORE);
   static constexpr int kOutBytes = kDirectStore ? 0 : kEpiWarps * 2 * 2048;
   static constexpr int kStagesRaw = (kSmemBudget - kOutBytes) / kStageBytes;
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
@@ -126,6 +139,24 @@ struct KParams {
   unsigned* err;
   uint64_t timeout_ns;
 };
+
+// Coordinates of cluster tile ct: its M tile group and its N tile.  Tiles are
+// visited in groups of kGroup M tile groups (the last group may be smaller),
+// M fastest within a group.
+__device__ __forceinline__ void tile_coords(int ct, int groups_m, int tiles_n, int* mg, int* nb) {
+  constexpr int kGroup = QLIN_GROUP_M;
+  if (kGroup <= 0) {
+    *nb = ct / groups_m;
+    *mg = ct % groups_m;
+    return;
+  }
+  const int per = kGroup * tiles_n;
+  const int grp = ct / per;
+  const int within = ct - grp * per;
+  const int gm = min(kGroup, groups_m - grp * kGroup);
+  *mg = grp * kGroup + within % gm;
+  *nb = within / gm;
+}
 
 // Bounded wait that ignores the abort flag: used to drain copies and MMAs in
 // flight before the CTA releases TMEM and exits.
@@ -173,8 +204,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
   uint8_t* out_stage = smem + C::kStages * C::kStageBytes;   // epilogue staging boxes
   uint64_t* full = reinterpret_cast<uint64_t*>(out_stage + C::kOutBytes);
   uint64_t* empty = full + C::kStages;
-  uint64_t* sf_ready = empty + C::kStages;   // NVFP4: the stage's scales are in TMEM
-  uint64_t* sf_full = sf_ready + C::kStages;  // NVFP4: the stage's scale bytes landed
+  uint64_t* sf_full = empty + C::kStages;   // NVFP4: the stage's scale bytes landed
   uint64_t* tmem_full = sf_full + C::kStages;
   uint64_t* tmem_empty = tmem_full + 2;
   uint64_t* mma_done = tmem_empty + 2;
@@ -189,9 +219,10 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
-      mbar_init(&full[s], 1);
+      // NVFP4: the scale-copy warps' commits (one per warp) also arrive on
+      // full, so the MMA issuer waits on one barrier per stage
+      mbar_init(&full[s], kFp4 ? 1 + C::kCpWarps : 1);
       mbar_init(&empty[s], 1);
-      mbar_init(&sf_ready[s], C::kCpWarps);   // one commit per scale-copy warp
       mbar_init(&sf_full[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -263,8 +294,9 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
       uint32_t phase = 0;
       int issued = 0;
       for (int ct = cid; ct < num_ctiles; ct += ncl) {
-        const int nb = ct / groups_m;
-        const int mb = (ct % groups_m) * kCM + rank;
+        int mg, nb;
+        tile_coords(ct, groups_m, tiles_n, &mg, &nb);
+        const int mb = mg * kCM + rank;
         bool ok = true;
         for (int kb = 0; kb < num_kb; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, ctl)) {
@@ -273,6 +305,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
           }
           uint8_t* sA = smem + stage * C::kStageBytes;
           uint8_t* sB = sA + C::kABytes;
+          uint8_t* sSF = sB + C::kBBytes;   // the stage's scale atoms: A's, then W's
           if (leader && pl == 0)
             mbar_arrive_expect_tx(&full[stage], kCM * (C::kABytes + C::kBBytes));
           if (kFp4 && leader && pl == kOpLanes)
@@ -289,9 +322,9 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
             c0 = kb * kRowBytes; c1 = nb * kBN + rank * (kBN / kCM) + part * kBRowsPart;
             c2 = 0; c3 = 0;
           } else if (pl == kOpLanes) {      // A scale atoms of this stage
-            dst = sB + C::kBBytes; c0 = kb * kStepsPerStage * 64; c1 = mb; c2 = 0; c3 = 0;
+            dst = sSF; c0 = kb * kStepsPerStage * 64; c1 = mb; c2 = 0; c3 = 0;
           } else {                          // W scale atoms (all atom rows of the N tile)
-            dst = sB + C::kBBytes + C::kSfaBytes; c0 = kb * kStepsPerStage * 64;
+            dst = sSF + C::kSfaBytes; c0 = kb * kStepsPerStage * 64;
             c1 = (nb * kBN) >> 7; c2 = 0; c3 = 0;   // first 128-row atom of the N tile
           }
           const uint32_t bar = bar0 + (uint32_t)(stage * 8);
@@ -327,11 +360,9 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
       const uint32_t idesc = kFp4    ? idesc_nvfp4(kBN, kMmaM)
                              : kBf16 ? (p.fp16 ? idesc_fp16(kBN, kMmaM) : idesc_bf16(kBN, kMmaM))
                                      : idesc_fp8(kBN, kMmaM);
-      // A stage is ready for its MMAs once its operands have landed (full)
-      // and, for NVFP4, its scales are in TMEM (sf_ready).
-      auto wait_ready = [&](int st, uint32_t ph) {
-        return mbar_wait(&full[st], ph, ctl) && (!kFp4 || mbar_wait(&sf_ready[st], ph, ctl));
-      };
+      // A stage is ready for its MMAs once its operands have landed and, for
+      // NVFP4, its scales are in TMEM (one barrier counts both).
+      auto wait_ready = [&](int st, uint32_t ph) { return mbar_wait(&full[st], ph, ctl); };
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
@@ -341,8 +372,11 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
         // 64-wide tiles use one half of a 128-row W scale atom: its rows
         // 32 w + lane sit in TMEM column w, so the odd tile's half starts two
         // columns in
-        const uint32_t sfb_off = kBN < 128 ? 2u * (uint32_t)((ct / groups_m) & 1) : 0u;
-        if (!mbar_wait(&tmem_empty[acc], acc_phase ^ 1u, ctl) || !wait_ready(stage, phase)) break;
+        int mg_, nb_;
+        tile_coords(ct, groups_m, tiles_n, &mg_, &nb_);
+        const uint32_t sfb_off = kBN < 128 ? 2u * (uint32_t)(nb_ & 1) : 0u;
+        if (!mbar_wait(&tmem_empty[acc], acc_phase ^ 1u, ctl)) break;
+        if (!wait_ready(stage, phase)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * kBN);
         for (int kb = 0; kb < num_kb; ++kb) {
@@ -383,7 +417,10 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
           } else {
             for (int jj = 0; jj < nsteps; ++jj) issue(jj, (jj > 0 || kb > 0) ? 1u : 0u);
           }
-          // the stage is free once the MMAs have read it (both CTAs' halves)
+          // The stage is free once the MMAs have read it (both CTAs' halves).
+          // The release comes right after the stage's last MMA: deferring it
+          // under the next stage's first MMA (to shorten the gap between
+          // issues) measured slower, the load pipeline being the bound.
           if (kPair)
             tc_commit_pair_mc(&empty[stage], kMask);
           else
@@ -392,8 +429,10 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
             stage = 0;
             phase ^= 1u;
           }
-          // the tile's next stage (an MMA issue blocks until the queue, about
-          // two MMAs deep, has room, so this wait overlaps the queued MMAs)
+          // the tile's next stage: one barrier test per stage (the scale
+          // copies arrive on the same barrier as the operands; a second
+          // barrier's test cost ~100 cycles a stage in shared memory this
+          // busy, the MMA queue holding about one instruction)
           if (kb + 1 < num_kb) {
             if (!wait_ready(stage, phase)) {
               ok = false;
@@ -458,18 +497,21 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
               tc_cp_scales(sfa_t, sdesc_scales(sSFA + j * 512));
 #pragma unroll
             for (int r = 0; r < C::kSfbAtoms; ++r) {
+              const uint32_t src = sSFB + r * kStepsPerStage * 512 + j * 512;
               if (kPair)
-                tc_cp_scales_pair(sfa_t + 4 + 4 * r,
-                                  sdesc_scales(sSFB + r * kStepsPerStage * 512 + j * 512));
+                tc_cp_scales_pair(sfa_t + 4 + 4 * r, sdesc_scales(src));
               else
-                tc_cp_scales(sfa_t + 4 + 4 * r,
-                             sdesc_scales(sSFB + r * kStepsPerStage * 512 + j * 512));
+                tc_cp_scales(sfa_t + 4 + 4 * r, sdesc_scales(src));
             }
           }
+          // the stage is ready for its MMAs once these copies and its
+          // operands have landed: both arrive on its full barrier.  (Its
+          // previous phase has completed: the scale boxes of this stage were
+          // issued after the MMAs of the stage that last used it.)
           if (kPair)
-            tc_commit_pair_mc(&sf_ready[stage], 1);
+            tc_commit_pair_mc(&full[stage], 1);
           else
-            tc_commit(&sf_ready[stage]);
+            tc_commit(&full[stage]);
           if (++stage == C::kStages) {
             stage = 0;
             phase ^= 1u;
@@ -504,10 +546,13 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
     for (int ct = cid; ct < num_ctiles; ct += ncl) {
       if (!mbar_wait(&tmem_full[acc], acc_phase, ctl)) break;
       tc_fence_after();
-      const int nb = ct / groups_m;
-      const int mb = (ct % groups_m) * kCM + rank;
+      int mg, nb;
+      tile_coords(ct, groups_m, tiles_n, &mg, &nb);
+      const int mb = mg * kCM + rank;
       const int64_t row = (int64_t)mb * kBM + quarter * 32 + lane;
+      // chunk c (32 columns) of this thread starts at column ccol(c)
       const int64_t col0 = (int64_t)nb * kBN + half * kCols;
+      auto ccol = [&](int c) -> int64_t { return col0 + c * 32; };
       uint32_t packed[kCols / 2];
       const uint32_t taddr =
           tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * kBN + half * kCols);
@@ -518,6 +563,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
       // 12 warps, 128 above) allows.
       constexpr int kBatch =
           (C::kNumAcc == 1 && C::kThreads <= 384) ? kChunks : (kChunks < 2 ? kChunks : 2);
+      static_assert(kChunks % kBatch == 0, "TMEM is released after the last batch");
 #pragma unroll
       for (int cb = 0; cb < kChunks; cb += kBatch) {
         uint32_t r[kBatch][32];
@@ -548,7 +594,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
 #pragma unroll
             for (int i = 0; i < 32; ++i) a[i] = alpha;
           } else {
-            const int64_t n0 = col0 + c * 32;
+            const int64_t n0 = ccol(c);
             if (p.w_per_channel && n0 < p.N) {
               const float4* sw = reinterpret_cast<const float4*>(p.sdec_w + n0);
 #pragma unroll
@@ -597,11 +643,11 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
         // columns (64 bytes) per chunk; N % 64 == 0, so a chunk is wholly
         // inside or outside the matrix
         if (p.y != nullptr && row < p.M) {
-          uint16_t* const yrow = p.y + row * p.N + col0;
+          uint16_t* const yrow = p.y + row * p.N;
 #pragma unroll
           for (int c = 0; c < kChunks; ++c) {
-            if (col0 + c * 32 >= p.N) break;
-            uint32_t* const dst = reinterpret_cast<uint32_t*>(yrow + c * 32);
+            if (ccol(c) >= p.N) continue;
+            uint32_t* const dst = reinterpret_cast<uint32_t*>(yrow + ccol(c));
             if (p.y_v8) {
               st_global_v8(dst, &packed[c * 16]);
               st_global_v8(dst + 8, &packed[c * 16 + 8]);
@@ -631,7 +677,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
-            tma_store_2d(&tmap_y, bufp, (int32_t)(col0 + c * 32), (int32_t)(row - lane));
+            tma_store_2d(&tmap_y, bufp, (int32_t)ccol(c), (int32_t)(row - lane));
             bulk_commit_group();
           }
         }
@@ -642,7 +688,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
           // bf16(y) * S_enc per element, 64 columns per group
 #pragma unroll
           for (int g = 0; g < kCols / 64; ++g) {
-            const int64_t c64 = col0 + g * 64;
+            const int64_t c64 = ccol(2 * g);   // chunks 2g, 2g + 1: 64 contiguous columns
             if (c64 < p.rq_col0 || c64 + 64 > p.rq_col0 + p.rq_cols || c64 >= p.N) continue;
             uint8_t* cp = p.rq_codes + row * p.rq_cols + (c64 - p.rq_col0);
 #pragma unroll
@@ -662,7 +708,7 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
         if (kRequant && kFp4) {
 #pragma unroll
           for (int g = 0; g < kCols / 64; ++g) {
-            const int64_t c64 = col0 + g * 64;
+            const int64_t c64 = ccol(2 * g);   // chunks 2g, 2g + 1: 64 contiguous columns
             if (c64 < p.rq_col0 || c64 + 64 > p.rq_col0 + p.rq_cols || c64 >= p.N) continue;
             const int64_t lc = c64 - p.rq_col0;
             uint32_t words[8];
@@ -886,9 +932,10 @@ cudaError_t dispatch_bn(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned
   // groups need 128-column tiles).
   const int64_t tiles_m = (a.M + kBM - 1) / kBM;
   const bool wide = tiles_m * ((a.N + 255) / 256) >= num_sms;
-  if (a.next_scale != nullptr)
+  if (a.next_scale != nullptr) {
     return wide ? launch_cfg<kFp4, 256, true, true>(a, s, num_sms, err, timeout_ns)
                 : launch_cfg<kFp4, 128, false, true>(a, s, num_sms, err, timeout_ns);
+  }
   if (wide) return launch_cfg<kFp4, 256, true, false>(a, s, num_sms, err, timeout_ns);
   const bool narrow = 2 * tiles_m * ((a.N + 127) / 128) <= num_sms;
   return narrow ? launch_cfg<kFp4, 64, false, false>(a, s, num_sms, err, timeout_ns)
