@@ -17,7 +17,9 @@ extern "C" {
  * `iters` back-to-back tcgen05.mma instructions from one thread, with its
  * operands resident in shared memory.
  *   kind  4 = NVFP4 (kind::mxf4nvf4, scale_vec::4X, K = 64 per instruction),
- *         8 = FP8 E4M3 (kind::f8f6f4, K = 32), 16 = bf16 (kind::f16, K = 16)
+ *         8 = FP8 E4M3 (kind::f8f6f4, K = 32), 16 = bf16 (kind::f16, K = 16);
+ *         kind + 100: the same with the A operand read from TMEM (written
+ *         there first by tcgen05.st) instead of shared memory
  *   pair  0 = cta_group::1 (M = 128), 1 = cta_group::2 (M = 256 on two SMs)
  *   n     the instruction's N: 256 for every kind, or 128 for kind 4, pair 0
  *   out   device array of 2 x (number of MMA-issuing CTAs) uint64: per issuing

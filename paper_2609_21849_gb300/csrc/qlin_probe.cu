@@ -5,9 +5,12 @@
 // also reported against, in FLOP per SM cycle (clock-independent) and in
 // FLOP/s at the clock the probe ran at.
 //
-// Only the instruction forms the GEMMs issue are used: kind::mxf4nvf4
+// The instruction kinds are the ones the GEMMs issue: kind::mxf4nvf4
 // block_scale scale_vec::4X (NVFP4), kind::f8f6f4 (E4M3) and kind::f16
-// (bf16), each as cta_group::1 (M = 128) and cta_group::2 (M = 256).
+// (bf16), each as cta_group::1 (M = 128) and cta_group::2 (M = 256), with A
+// in shared memory (as in the GEMMs) or in TMEM (the A-from-tensor-memory
+// form, A written there by tcgen05.st), which shows whether operand reads
+// from shared memory bound the rate.
 #include <cstdio>
 
 #include "qlin_device.cuh"
@@ -44,9 +47,56 @@ __device__ __forceinline__ bool probe_wait(uint64_t* bar, uint32_t parity, unsig
   return false;
 }
 
+// A operand in TMEM: D[tmem] (+)= A[tmem] * B[smem]^T.
+__device__ __forceinline__ void mma_ts(int kind, bool pair, uint32_t d, uint32_t a_t, uint64_t b,
+                                       uint32_t idesc, uint32_t sfa, uint32_t sfb, uint32_t acc) {
+  if (kind == 4 && pair)
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::2.kind::mxf4nvf4.block_scale.scale_vec::4X"
+                 " [%0], [%1], %2, %3, [%5], [%6], p;\n\t}" ::"r"(d),
+                 "r"(a_t), "l"(b), "r"(idesc), "r"(acc), "r"(sfa), "r"(sfb) : "memory");
+  else if (kind == 4)
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::mxf4nvf4.block_scale.scale_vec::4X"
+                 " [%0], [%1], %2, %3, [%5], [%6], p;\n\t}" ::"r"(d),
+                 "r"(a_t), "l"(b), "r"(idesc), "r"(acc), "r"(sfa), "r"(sfb) : "memory");
+  else if (kind == 8 && pair)
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+                 "r"(a_t), "l"(b), "r"(idesc), "r"(acc) : "memory");
+  else if (kind == 8)
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+                 "r"(a_t), "l"(b), "r"(idesc), "r"(acc) : "memory");
+  else if (pair)
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+                 "r"(a_t), "l"(b), "r"(idesc), "r"(acc) : "memory");
+  else
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+                 "r"(a_t), "l"(b), "r"(idesc), "r"(acc) : "memory");
+}
+
+// Write 32 consecutive TMEM columns of this thread's lane.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0],"
+      " {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16,"
+      " %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+
 // kKind: 4 = NVFP4 (mxf4nvf4, K = 64), 8 = FP8 (f8f6f4, K = 32), 16 = bf16
 // (f16, K = 16); every instruction reads 32 bytes of K per operand row.
-template <int kKind, bool kPair, int kN>
+// kATmem: A from TMEM columns [384, 416) (8 columns per instruction).
+template <int kKind, bool kPair, int kN, bool kATmem = false>
 __global__ void __launch_bounds__(kProbeThreads, 1)
     mma_probe_kernel(int iters, unsigned long long* out, unsigned* err) {
   extern __shared__ uint8_t smem_raw[];
@@ -86,6 +136,24 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
     __syncthreads();
   tc_fence_after();
   const uint32_t tb = tmem_slot;
+  if (kATmem) {
+    // A in TMEM: each warp writes its lane quarter's 32 columns
+    uint32_t r[32];
+    for (int i = 0; i < 32; ++i) {
+      uint32_t v = hash32((uint32_t)(threadIdx.x * 32 + i) * 2246822519u + blockIdx.x);
+      if (kKind == 8) v &= 0xBFBFBFBFu;
+      if (kKind == 16) v &= 0xBFFFBFFFu;
+      r[i] = v;
+    }
+    tmem_st32(tb + ((uint32_t)((threadIdx.x >> 5) * 32) << 16) + 384, r);
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    tc_fence_before();
+    if (kPair)
+      cluster_sync();
+    else
+      __syncthreads();
+    tc_fence_after();
+  }
   if (threadIdx.x == 0 && rank == 0) {
     constexpr int kM = kPair ? 256 : 128;
     const uint32_t idesc = kKind == 4 ? idesc_nvfp4(kN, kM)
@@ -113,7 +181,9 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
       const uint32_t j = (uint32_t)(i & 3) * 32;
       const uint64_t ad = sdesc_k128(a + j), bd = sdesc_k128(b + j);
       const uint32_t acc = i > 0 ? 1u : 0u;
-      if (kKind == 4) {
+      if (kATmem) {
+        mma_ts(kKind, kPair, tb, tb + 384 + (uint32_t)(i & 3) * 8, bd, idesc, sf_t, sf_t + 4, acc);
+      } else if (kKind == 4) {
         if (kPair)
           mma_nvfp4_pair(tb, ad, bd, idesc, sf_t, sf_t + 4, acc);
         else
@@ -155,10 +225,10 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
   }
 }
 
-template <int kKind, bool kPair, int kN>
+template <int kKind, bool kPair, int kN, bool kATmem = false>
 cudaError_t launch_probe(int ctas, int iters, unsigned long long* out, unsigned* err,
                          cudaStream_t s) {
-  auto kern = mma_probe_kernel<kKind, kPair, kN>;
+  auto kern = mma_probe_kernel<kKind, kPair, kN, kATmem>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        kProbeSmem);
   if (e != cudaSuccess) return e;
@@ -184,6 +254,9 @@ using namespace qlin;
 
 extern "C" int qlin_probe_mma(int kind, int pair, int n, int ctas, int iters,
                               unsigned long long* out, unsigned* err, void* stream) {
+  // kind + 100: the same kind with A in TMEM
+  const bool a_tmem = kind > 100;
+  if (a_tmem) kind -= 100;
   if (out == nullptr || err == nullptr || iters < 1 || ctas < 1) return 1;
   if (pair && ctas % 2 != 0) return 1;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -192,7 +265,8 @@ extern "C" int qlin_probe_mma(int kind, int pair, int n, int ctas, int iters,
 #define QLIN_PROBE_CASE(K, P, N)                                      \
   if (kind == K && (pair != 0) == P && n == N) {                      \
     matched = true;                                                   \
-    e = launch_probe<K, P, N>(ctas, iters, out, err, s);              \
+    e = a_tmem ? launch_probe<K, P, N, true>(ctas, iters, out, err, s) \
+               : launch_probe<K, P, N, false>(ctas, iters, out, err, s); \
   }
   QLIN_PROBE_CASE(4, true, 256);
   QLIN_PROBE_CASE(4, false, 256);

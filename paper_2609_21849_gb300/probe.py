@@ -20,13 +20,18 @@ from . import build
 
 _lib = None
 
-# (name, kind, pair, n, K per instruction)
+# (name, kind, pair, n, K per instruction); kind + 100: A read from TMEM
 CASES = (("nvfp4_pair_256x256x64", 4, 1, 256, 64),
          ("nvfp4_cta_128x256x64", 4, 0, 256, 64),
          ("nvfp4_cta_128x128x64", 4, 0, 128, 64),
          ("fp8_pair_256x256x32", 8, 1, 256, 32),
          ("fp8_cta_128x256x32", 8, 0, 256, 32),
-         ("bf16_pair_256x256x16", 16, 1, 256, 16))
+         ("bf16_pair_256x256x16", 16, 1, 256, 16),
+         ("nvfp4_pair_256x256x64_a_tmem", 104, 1, 256, 64),
+         ("nvfp4_cta_128x256x64_a_tmem", 104, 0, 256, 64),
+         ("nvfp4_cta_128x128x64_a_tmem", 104, 0, 128, 64),
+         ("fp8_pair_256x256x32_a_tmem", 108, 1, 256, 32),
+         ("bf16_pair_256x256x16_a_tmem", 116, 1, 256, 16))
 
 
 def _load():
