@@ -551,6 +551,34 @@ def measure_headline_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak
                                    "frac_of_bound": round(bound / t, 3),
                                    "bound": "bytes" if nbytes / (hbm * 1e9) > fl / (peak * 1e12) else "compute"}
     out["a8_small_m"] = res
+
+    # ---- the translator MLP forward (Sec. 3's d3072 translator: 512 tokens,
+    # 1024 -> 3072 -> 2560; dynamic input quantization, the first linear's
+    # epilogue re-quantizing the hidden activations), one CUDA graph per
+    # format, against the sum of its three kernels' max(compute, bytes) bounds
+    from paper_2609_21849_gb300 import translator
+    xt, w1t, w2t = synthetic.translator_mlp()
+    xtd = to_dev(xt, torch)
+    Mt, Kt = xt.shape
+    Ht, Ot = w1t.shape[0], w2t.shape[0]
+    tr = {}
+    for fmt in ("nvfp4", "fp8"):
+        t = translator.build_translator(fmt, w1t, w2t, Mt)
+        t.calibrate(xtd)
+        tm = g_time(torch, stream, lambda t=t: t.forward(xtd, stream), 20)
+        qb = 0.5625 if fmt == "nvfp4" else 1.0          # bytes per quantized element
+        peak = fp4_peak if fmt == "nvfp4" else fp8_peak
+        f1, f2 = 2 * Mt * Ht * Kt, 2 * Mt * Ot * Ht
+        b0 = Mt * Kt * (2 + qb)                          # quantizer: read x, write x_q
+        b1 = (Mt * Kt + Ht * Kt + Mt * Ht) * qb          # x_q, W1 in; h_q out
+        b2 = (Mt * Ht + Ot * Ht) * qb + Mt * Ot * 2      # h_q, W2 in; bf16 y out
+        bound = (b0 / (hbm * 1e9) + max(f1 / (peak * 1e12), b1 / (hbm * 1e9))
+                 + max(f2 / (peak * 1e12), b2 / (hbm * 1e9)))
+        tr[fmt] = {"us": round(tm * 1e6, 2), "TFLOP/s": round(t.flops / tm / 1e12, 1),
+                   "bound_us": round(bound * 1e6, 3), "frac_of_bound": round(bound / tm, 3),
+                   "launches": 3, "note": "one forward per graph node group, weights L2-warm"}
+        del t
+    out["f4_translator_mlp"] = tr
     return out
 
 

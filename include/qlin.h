@@ -271,17 +271,21 @@ qlin_status qlin_gemm_fp16(const void *a_fp16, int64_t lda, const void *w_fp16, 
  * run-time activation quantization, here with the tensor scale of the layer's
  * own output instead of a calibrated one):
  *   y = A W^T (bf16, as qlin_gemm_nvfp4), while the GEMM epilogue reduces
- *   amax(|y|) into a workspace word; then y_q = NVFP4(y) with the dynamic
- *   S_dec = amax / 2688 (1 if amax == 0), exactly as
+ *   amax(|y|) into a workspace word and the GEMM's last CTA turns it into
+ *   the dynamic S_dec = amax / 2688 (1 if amax == 0), written to
+ *   y_q->tensor_scale; then y_q = NVFP4(y) with that scale, exactly as
  *   qlin_quantize_act_nvfp4(y, NULL) would produce it, without its amax pass
- *   over y.
+ *   over y.  y is stored with an L2 keep hint, since the quantizer reads it
+ *   right after.
  *  A, W:      NVFP4 operands as for qlin_gemm_nvfp4.
  *  y_bf16:    bf16 [A->rows, W->rows], 16-byte aligned (required: the
  *             quantizer reads it).
  *  y_q:       rows == A->rows, K == W->rows; codes, scales and tensor_scale
  *             are written.
- *  workspace: as for qlin_quantize_act_nvfp4 (one word of it is cleared and
- *             used per call).
+ *  workspace: as for qlin_quantize_act_nvfp4: zero-filled before its first
+ *             use, left zero-filled by every call (two of its words count
+ *             within a call); calls that share one workspace must not
+ *             overlap on the GPU.
  * Errors: INVALID_ARG, MISALIGNED, WORKSPACE, CUDA.
  */
 qlin_status qlin_linear_dynamic(const qlin_nvfp4_t *A, const qlin_nvfp4_t *W, void *y_bf16,

@@ -122,7 +122,9 @@ qlin_status check_workspace(void* ws, size_t ws_bytes) {
 // two-pass route (cleared before each use).
 constexpr int kWsOnePass = 0;
 constexpr int kWsTwoPassAmax = 4;
-constexpr int kWsChainAmax = 5;   // qlin_linear_dynamic: max |y| from the GEMM epilogue
+// qlin_linear_dynamic: max |y| from the GEMM epilogue and the epilogue's
+// departure count (words 5 and 6; zero between calls)
+constexpr int kWsChainAmax = 5;
 
 // Dynamic NVFP4 activation quantization: one read of x when it fits on chip,
 // else the amax pass then the quantizer.  clear: zero the one-read words first.
@@ -251,9 +253,11 @@ qlin_status qlin_quantize_weight(const void* w_bf16, int64_t N, int64_t K, qlin_
 static qlin_status gemm_common(bool fp4, const void* Aany, const void* Wany, void* y,
                                const float* next_scale, qlin_nvfp4_t* y_q, int64_t rq_col0,
                                void* stream, unsigned* y_amax = nullptr,
-                               qlin_fp8_t* y_q8 = nullptr) {
+                               qlin_fp8_t* y_q8 = nullptr, float* y_sdec = nullptr) {
   GemmArgs a{};
   a.y_amax = y_amax;
+  a.y_departures = y_amax != nullptr ? y_amax + 1 : nullptr;
+  a.y_sdec = y_sdec;
   a.fp4 = fp4;
   if (fp4) {
     const qlin_nvfp4_t* A = static_cast<const qlin_nvfp4_t*>(Aany);
@@ -318,8 +322,6 @@ static qlin_status gemm_common(bool fp4, const void* Aany, const void* Wany, voi
   unsigned* status;
   int sms;
   QLIN_TRY(device_state(&status, &sms));
-  if (y_amax != nullptr)
-    QLIN_CUDA(cudaMemsetAsync(y_amax, 0, sizeof(unsigned), static_cast<cudaStream_t>(stream)));
   cudaError_t e = launch_gemm(a, static_cast<cudaStream_t>(stream), sms, status,
                               g_timeout_ns.load(std::memory_order_relaxed));
   if (e != cudaSuccess) return cuda_fail(e);
@@ -389,14 +391,16 @@ qlin_status qlin_linear_dynamic(const qlin_nvfp4_t* A, const qlin_nvfp4_t* W, vo
   QLIN_TRY(check_workspace(workspace, ws_bytes));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   unsigned* amax = static_cast<unsigned*>(workspace) + kWsChainAmax;
-  // y and its tensor amax in one GEMM (the word is cleared first), then the
-  // quantizer with that scale
-  QLIN_TRY(gemm_common(true, A, W, y_bf16, nullptr, nullptr, 0, stream, amax));
+  // y and its tensor scale in one GEMM (its last CTA writes S_dec into y_q's
+  // tensor scale and resets the scratch words), then the quantizer of y with
+  // that scale
+  QLIN_TRY(gemm_common(true, A, W, y_bf16, nullptr, nullptr, 0, stream, amax, nullptr,
+                       y_q->tensor_scale));
   unsigned* status;
   int sms;
   QLIN_TRY(device_state(&status, &sms));
-  QLIN_CUDA(launch_quant_nvfp4(y_bf16, A->rows, W->rows, reinterpret_cast<const float*>(amax),
-                               true, *y_q, s, sms, status, timeout()));
+  QLIN_CUDA(launch_quant_nvfp4(y_bf16, A->rows, W->rows, y_q->tensor_scale, false, *y_q, s, sms,
+                               status, timeout()));
   return QLIN_OK;
 }
 

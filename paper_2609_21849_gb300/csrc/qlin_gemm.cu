@@ -134,6 +134,8 @@ struct KParams {
   float* rq_tensor_scale;
   int64_t rq_col0, rq_cols;
   unsigned* y_amax;   // optional: max |bf16 y| over the output, as fp32 bits (atomicMax)
+  unsigned* y_departures;   // with y_amax: CTAs done (the last one turns the amax into S_dec)
+  float* y_sdec;            // with y_amax: where the last CTA writes S_dec = amax / 2688
   int fp16;           // 16-bit operand kernel only: fp16 operands and output (else bf16)
   int y_v8;           // y is 32-byte aligned: direct stores may use 32-byte vectors
   unsigned* err;
@@ -183,6 +185,21 @@ __device__ __forceinline__ void st_global_v4(void* p, uint32_t a, uint32_t b, ui
 __device__ __forceinline__ void st_global_v8(void* p, const uint32_t* v) {
   asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(v[0]),
                "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+               : "memory");
+}
+
+// The same stores with an L2 cache-policy hint (createpolicy result).
+__device__ __forceinline__ void st_global_v8_hint(void* p, const uint32_t* v, uint64_t pol) {
+  asm volatile("st.global.L2::cache_hint.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8}, %9;" ::"l"(
+                   p),
+               "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]),
+               "r"(v[7]), "l"(pol)
+               : "memory");
+}
+__device__ __forceinline__ void st_global_v4_hint(void* p, uint32_t a, uint32_t b, uint32_t c,
+                                                  uint32_t d, uint64_t pol) {
+  asm volatile("st.global.L2::cache_hint.v4.b32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "r"(a),
+               "r"(b), "r"(c), "r"(d), "l"(pol)
                : "memory");
 }
 
@@ -644,18 +661,32 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
         // inside or outside the matrix
         if (p.y != nullptr && row < p.M) {
           uint16_t* const yrow = p.y + row * p.N;
+          // With an output amax (the dynamic chain), y is read back right
+          // after this kernel by the quantizer: keep it in L2 if it can.
+          const bool keep = p.y_amax != nullptr;
+          const uint64_t pol = keep ? policy_evict_last() : 0ull;
 #pragma unroll
           for (int c = 0; c < kChunks; ++c) {
             if (ccol(c) >= p.N) continue;
             uint32_t* const dst = reinterpret_cast<uint32_t*>(yrow + ccol(c));
             if (p.y_v8) {
-              st_global_v8(dst, &packed[c * 16]);
-              st_global_v8(dst + 8, &packed[c * 16 + 8]);
+              if (keep) {
+                st_global_v8_hint(dst, &packed[c * 16], pol);
+                st_global_v8_hint(dst + 8, &packed[c * 16 + 8], pol);
+              } else {
+                st_global_v8(dst, &packed[c * 16]);
+                st_global_v8(dst + 8, &packed[c * 16 + 8]);
+              }
             } else {
 #pragma unroll
-              for (int k = 0; k < 4; ++k)
-                st_global_v4(dst + 4 * k, packed[c * 16 + 4 * k], packed[c * 16 + 4 * k + 1],
-                             packed[c * 16 + 4 * k + 2], packed[c * 16 + 4 * k + 3]);
+              for (int k = 0; k < 4; ++k) {
+                if (keep)
+                  st_global_v4_hint(dst + 4 * k, packed[c * 16 + 4 * k], packed[c * 16 + 4 * k + 1],
+                                    packed[c * 16 + 4 * k + 2], packed[c * 16 + 4 * k + 3], pol);
+                else
+                  st_global_v4(dst + 4 * k, packed[c * 16 + 4 * k], packed[c * 16 + 4 * k + 1],
+                               packed[c * 16 + 4 * k + 2], packed[c * 16 + 4 * k + 3]);
+              }
             }
           }
         }
@@ -747,6 +778,25 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
     // stores' global writes complete with the grid (as for any store), so
     // the CTA does not wait for them.
     if (lane == 0) bulk_wait_group_read<0>();
+    if (p.y_amax != nullptr) {
+      // The output's tensor scale: once every epilogue warp of the CTA has
+      // added its maxima, the CTA departs; the last CTA of the grid to depart
+      // turns the amax into S_dec = amax / (6 * 448) (1 for an all-zero
+      // output), writes it where the quantizer of y reads its scale, and
+      // resets both scratch words for the next call (so no clearing node
+      // precedes the kernel).
+      asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+      if (threadIdx.x == C::kEpiWarp0 * 32) {
+        __threadfence();
+        if (atomicAdd(p.y_departures, 1u) == gridDim.x - 1) {
+          __threadfence();
+          const unsigned bits = atomicExch(p.y_amax, 0u);
+          const float amax = __uint_as_float(bits);
+          *p.y_sdec = bits == 0u ? 1.0f : __fdiv_rn(amax, 2688.0f);
+          atomicExch(p.y_departures, 0u);
+        }
+      }
+    }
   }
 
   // No CTA of the cluster may exit while a peer can still multicast into it
@@ -881,6 +931,8 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   p.rq_col0 = a.rq_col0;
   p.rq_cols = a.rq_cols;
   p.y_amax = a.y_amax;
+  p.y_departures = a.y_departures;
+  p.y_sdec = a.y_sdec;
   p.fp16 = kBf16 && a.fp16 ? 1 : 0;
   p.y_v8 = (reinterpret_cast<uintptr_t>(a.y) & 31u) == 0 ? 1 : 0;
   p.err = err;

@@ -58,8 +58,12 @@ struct GemmArgs {
   uint8_t* rq_scales;
   float* rq_tensor_scale;
   int64_t rq_col0, rq_cols;
-  // optional max |bf16 y| (fp32 bits, atomicMax; cleared by the caller)
+  // optional max |bf16 y| (fp32 bits, atomicMax), with a departure count;
+  // both are zero at launch and reset by the last CTA, which writes
+  // S_dec = amax / (6 * 448) to y_sdec
   unsigned* y_amax;
+  unsigned* y_departures;
+  float* y_sdec;
 };
 cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned* err,
                         uint64_t timeout_ns);

@@ -16,8 +16,8 @@ Recipes (seed s):
         without replacement, are multiplied by 20.
       - "channel gain": x = z * g[k], g = exp(N(0, 1)) per channel k.
       - "channel outliers": round(0.01 * K) channels multiplied by 20.
-  * weights: rng = default_rng([s, 1]); w ~ N(0, sigma^2), drawn in the order
-    the weights are listed.
+  * weights: rng = default_rng([s, 1]) (the translator MLP: [s, 3]);
+    w ~ N(0, sigma^2), drawn in the order the weights are listed.
 """
 from __future__ import annotations
 
@@ -80,10 +80,10 @@ def act_normal(seed: int, M: int, K: int) -> np.ndarray:
     return bf16_bits(_normal(rng, (M, K)))
 
 
-def weights(seed: int, shapes, sigma: float):
+def weights(seed: int, shapes, sigma: float, stream: int = 1):
     """Weights [N, K] ~ N(0, sigma^2) for each (N, K) in ``shapes``, drawn in
-    order from default_rng([seed, 1]).  Yields bf16 bit arrays."""
-    rng = np.random.default_rng([seed, 1])
+    order from default_rng([seed, stream]).  Yields bf16 bit arrays."""
+    rng = np.random.default_rng([seed, stream])
     for (N, K) in shapes:
         yield bf16_bits(_normal(rng, (N, K), sigma))
 
@@ -119,6 +119,19 @@ def translator(M=512, seed=3):
     x2 = bf16_bits(_normal(np.random.default_rng([seed, 2]), (M, 2560)))
     w1, w2 = weights(seed, [(2560, 1024), (1024, 2560)], 0.03)
     return x1, x2, w1, w2
+
+
+TRANSLATOR_IN, TRANSLATOR_HIDDEN, TRANSLATOR_OUT = 1024, 3072, 2560
+
+
+def translator_mlp(M=512, seed=3):
+    """The d3072 translator MLP (0.6B encoder features -> 4B conditioning):
+    x [512, 1024] N(0, 1) (the translator linears' x1), W1 [3072, 1024] and
+    W2 [2560, 3072] N(0, 0.03^2) from default_rng([seed, 3])."""
+    x = act_normal(seed, M, TRANSLATOR_IN)
+    w1, w2 = weights(seed, [(TRANSLATOR_HIDDEN, TRANSLATOR_IN),
+                            (TRANSLATOR_OUT, TRANSLATOR_HIDDEN)], 0.03, stream=3)
+    return x, w1, w2
 
 
 STACK_LAYERS = (("qkv", 3 * HIDDEN, HIDDEN), ("out", HIDDEN, HIDDEN),
