@@ -46,7 +46,10 @@ def parse():
     ap.add_argument("--steps", type=int, default=16384)
     ap.add_argument("--warmup", type=int, default=32)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--no-rows", action="store_true", help="skip the secondary row measurements")
+    ap.add_argument("--no-rows", action="store_true",
+                    help="time the step only: skip the quantizer, GEMM, translator and secondary rows")
+    ap.add_argument("--sustained-s", type=float, default=1.0,
+                    help="seconds of step replay after the timed region for the clock samples (0: none)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     return ap.parse_args()
 
@@ -285,7 +288,8 @@ def run_ours(args, dist: Dist):
         gemm_s = timed(lambda: qlin.qlin_linear_fused(As[0], Wq[0], ys[0], next_scale, yqs[0]),
                        200, torch, stream)
     gemm_tflops = STEP_FLOPS / gemm_s / 1e12
-    sus_steps = S * max(1, int(1.0 / max(per_step, 1e-6)) // S)
+    sus_steps = (S * max(1, int(args.sustained_s / max(per_step, 1e-6)) // S)
+                 if args.sustained_s > 0 else 0)
     s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     s0.record(stream)
     sus_used = run_steps(sus_steps)
@@ -296,8 +300,9 @@ def run_ours(args, dist: Dist):
                      f"step graph right after it ({sus_steps} steps)")
     sus_sec = s0.elapsed_time(s1) / 1e3
     sus_gemm = [a.elapsed_time(b) / 1e3 for evs in sus_used for a, b in evs]
-    sustained = {"steps": sus_steps, "ms_per_step": round(sus_sec / sus_steps * 1e3, 5),
-                 "value": round(STEP_FLOPS * sus_steps / sus_sec / 1e12, 2),
+    sustained = {"steps": sus_steps,
+                 "ms_per_step": round(sus_sec / sus_steps * 1e3, 5) if sus_steps else None,
+                 "value": round(STEP_FLOPS * sus_steps / sus_sec / 1e12, 2) if sus_steps else None,
                  "gemm_us": round(statistics.mean(sus_gemm) * 1e6, 2) if sus_gemm else None}
 
     # ---- end to end through the public API with host buffers: every step
@@ -399,9 +404,9 @@ def run_ours(args, dist: Dist):
                      "algorithmic": f"{STEP_FLOPS / 1e9:.2f} GFLOP per launch; {gemm_s * 1e6:.2f} us avg launch"},
         "mma_probe": ceil,
     }
-    out.update(measure_headline_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak,
-                                     fp4_ceil, fp8_ceil))
     if not args.no_rows:
+        out.update(measure_headline_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak,
+                                         fp4_ceil, fp8_ceil))
         out["rows"] = measure_rows(torch, qlin, synthetic, stream, pk, fp4_peak, fp8_peak)
     del xs, As, ys, yqs, Wq
     torch.cuda.empty_cache()
