@@ -116,7 +116,7 @@ size_t qlin_workspace_size(int64_t M, int64_t K);
  *                first runs an amax pass over x.
  *  out:          rows == M, K == K; codes, scales and tensor_scale are written
  *                (tensor_scale receives S_dec in both modes).
- *  workspace:    device memory of >= qlin_workspace_size() bytes, 4-byte
+ *  workspace:    device memory of >= qlin_workspace_size() bytes, 8-byte
  *                aligned, zero-filled before its first use; every call leaves
  *                it zero-filled again (its words carry a grid-wide amax and
  *                arrival counts inside one call).  Used only in dynamic mode,

@@ -99,8 +99,10 @@ qlin_status check_fp8(const qlin_fp8_t* t, int64_t rows, int64_t K) {
 }
 
 qlin_status check_workspace(void* ws, size_t ws_bytes) {
-  if (ws == nullptr || ws_bytes < sizeof(unsigned)) return QLIN_ERR_WORKSPACE;
-  if (!aligned(ws, 4)) return QLIN_ERR_MISALIGNED;
+  if (ws == nullptr || ws_bytes < qlin_workspace_size(0, 0)) return QLIN_ERR_WORKSPACE;
+  // 8-byte aligned: the one-read quantizer reads its amax and arrival words
+  // as one 64-bit load
+  if (!aligned(ws, 8)) return QLIN_ERR_MISALIGNED;
   return QLIN_OK;
 }
 

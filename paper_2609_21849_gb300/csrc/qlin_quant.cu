@@ -439,9 +439,11 @@ constexpr int kOnePassSliceMax = 14 * 1024;       // chunks: 224 KB of data at m
 // NVFP4 steps of run_slice: two 2-chunk units per thread and step
 constexpr int kOnePassSteps = (kOnePassSliceMax + 4 * kOnePassThreads - 1) / (4 * kOnePassThreads);
 
-__device__ __forceinline__ uint32_t ld_acquire_gpu(const unsigned* p) {
-  uint32_t v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+// The amax word and the arrival count as one 64-bit acquire load (they are
+// adjacent words of one 8-byte-aligned pair, low word first).
+__device__ __forceinline__ uint64_t ld_acquire_gpu_pair(const unsigned* p) {
+  uint64_t v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
   return v;
 }
 
@@ -521,15 +523,20 @@ __global__ void __launch_bounds__(kOnePassThreads, 1)
     if (b) atomicMax(&sync[0], b << 16);
     // the arrival releases the maximum above to every CTA that sees it
     asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(&sync[1]) : "memory");
+    // The count and the amax are read together: a load that sees every
+    // CTA's arrival also sees every maximum released before it, which saves
+    // the second round trip to L2 that reading the amax afterwards took.
     const uint64_t t0 = global_timer_ns();
-    while (ld_acquire_gpu(&sync[1]) < gridDim.x) {
+    uint64_t pair = ld_acquire_gpu_pair(&sync[0]);
+    while ((uint32_t)(pair >> 32) < gridDim.x) {
       if (global_timer_ns() - t0 > timeout_ns) {
         atomicExch(err, kErrTimeout);
         abort_flag = 1;
         break;
       }
+      pair = ld_acquire_gpu_pair(&sync[0]);
     }
-    s_amax = __uint_as_float(ld_acquire_gpu(&sync[0]));
+    s_amax = __uint_as_float((uint32_t)pair);
   }
   __syncthreads();
   if (tid == 0) {

@@ -75,8 +75,13 @@ def test_argument_errors_return_before_launch(lib):
     assert lib.qlin_quantize_act_nvfp4(16, 64, 256, None, ctypes.byref(d), 16, 256, None) == 1
     # misaligned input pointer
     assert lib.qlin_quantize_act_nvfp4(24, 128, 256, None, ctypes.byref(d), 16, 256, None) == 3
-    # dynamic scale without workspace
+    # dynamic scale without workspace, with one smaller than qlin_workspace_size(), and with
+    # one only 4-byte aligned (its first two words are read as one 64-bit load)
     assert lib.qlin_quantize_act_nvfp4(16, 128, 256, None, ctypes.byref(d), None, 0, None) == 6
+    assert lib.qlin_quantize_act_nvfp4(16, 128, 256, None, ctypes.byref(d), 16, 28, None) == 6
+    assert lib.qlin_quantize_act_nvfp4(16, 128, 256, None, ctypes.byref(d), 20, 256, None) == 3
+    f8 = qlin.FP8Desc(16, 16, 128, 256, 0)
+    assert lib.qlin_quantize_act_fp8(16, 128, 256, None, ctypes.byref(f8), 20, 256, None) == 3
     # GEMM: K mismatch, N not a multiple of 64, nothing to write
     a = qlin.NVFP4Desc(16, 16, 16, 128, 256)
     w = qlin.NVFP4Desc(16, 16, 16, 256, 512)
