@@ -12,7 +12,7 @@
 //          drives both SMs' tensor cores; each CTA holds its own 128 rows of A
 //          and its own half of the W tile in shared memory.
 //   single 128 x 128 tiles on one CTA, for small M (the translator's linears).
-// Roles (one persistent CTA per SM; 12 warps, 13 for NVFP4 pair tiles):
+// Roles (one persistent CTA per SM; 12 warps, 15 for NVFP4 pair tiles):
 //   warp 0      TMA producer: per pipeline stage one 4-D tensor copy per lane,
 //               the A tile and the W tile from two lanes as one instruction
 //               (and, except for NVFP4 pair tiles, the A and W scale atoms
@@ -22,9 +22,10 @@
 //               NVFP4 kind::mxf4nvf4 scale_vec::4X with K = 64, FP8
 //               kind::f8f6f4 with K = 32, bf16 / fp16 kind::f16 with K = 16)
 //               into an fp32 TMEM accumulator.
-//   warps 2, 3  NVFP4: block scales shared -> TMEM (tcgen05.cp), beside the
-//               MMA stream, each warp the atoms of half the stage's MMA steps.
-//   warp 4      NVFP4 pair tiles: TMA producer of the scale atoms.
+//   warps 2..   NVFP4: block scales shared -> TMEM (tcgen05.cp), beside the
+//               MMA stream (two warps, four for pair tiles), each warp the
+//               atoms of an equal share of the stage's MMA steps.
+//   next warp   NVFP4 pair tiles: TMA producer of the scale atoms.
 //   last 8      epilogue: tcgen05.ld of the accumulator, alpha, 16-bit
 //               rounding; pair tiles store y straight from registers (FP8 /
 //               16-bit tiles use the freed staging memory for a seventh
@@ -49,7 +50,7 @@ constexpr int kEpiWarps = 8;
 // of NVFP4 pair tiles, a warp of its own for their scale boxes, and row boxes
 // per operand tile and stage.
 #ifndef QLIN_PAIR_CP_WARPS
-#define QLIN_PAIR_CP_WARPS 2
+#define QLIN_PAIR_CP_WARPS 4
 #endif
 #ifndef QLIN_SPLIT_SCALE_ISSUE
 #define QLIN_SPLIT_SCALE_ISSUE 1
@@ -483,8 +484,12 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
     // each scale-copy warp), beside the MMA stream: a tcgen05.cp occupies its
     // issuing thread ~80-120 cycles while the MMAs run, and a stage needs 12
     // (pair tiles), so each warp copies the atoms of an equal share of the
-    // stage's MMA steps.  In a pair, CTA 0's copies fill both SMs' TMEM from
-    // their own shared memory.
+    // stage's MMA steps.  Copies issued from separate warps overlap (12 take
+    // ~850 cycles from two warps, ~510 from four, with the MMAs running: the
+    // MMAs' rate is unaffected), so pair tiles use four.  (A converged
+    // instruction from several lanes of one warp does not issue one copy per
+    // lane.)  In a pair, CTA 0's copies fill both SMs' TMEM from their own
+    // shared memory.
     if (kFp4 && lane == 0 && leader) {
       const int sw = warp - 2;
       int stage = 0;
