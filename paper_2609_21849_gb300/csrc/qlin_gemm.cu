@@ -14,10 +14,11 @@
 //   single 128 x 128 tiles on one CTA, for small M (the translator's linears).
 // Roles (one persistent CTA per SM; 12 warps, 15 for NVFP4 pair tiles):
 //   warp 0      TMA producer: per pipeline stage one 4-D tensor copy per lane,
-//               the A tile and the W tile from two lanes as one instruction
-//               (and, except for NVFP4 pair tiles, the A and W scale atoms
-//               from two more lanes).  In a pair, CTA 1's copies complete on
-//               CTA 0's barriers (cta_group::2 form).
+//               the A tile and the W tile as two row boxes each from four
+//               lanes, as one instruction (and, except for NVFP4 pair tiles,
+//               the A and W scale atoms from two more lanes).  In a pair,
+//               CTA 1's copies complete on CTA 0's barriers (cta_group::2
+//               form).
 //   warp 1      TMEM allocation; MMA issue (per 32 bytes of K one tcgen05.mma:
 //               NVFP4 kind::mxf4nvf4 scale_vec::4X with K = 64, FP8
 //               kind::f8f6f4 with K = 32, bf16 / fp16 kind::f16 with K = 16)
@@ -87,6 +88,7 @@ struct Cfg {
   // consecutive warps cover the accumulator).  NVFP4 pair tiles need 12
   // scale copies per stage, shared between the scale-copy warps.
   static constexpr int kCpWarps = (kFp4 && kPair) ? QLIN_PAIR_CP_WARPS : 2;
+  static_assert(kStepsPerStage % kCpWarps == 0, "each scale-copy warp takes whole MMA steps");
   // NVFP4 pair tiles: a warp of its own issues the scale boxes, so the
   // operand boxes' instruction has two lanes instead of four
   static constexpr int kScaleWarp = (kFp4 && kPair && QLIN_SPLIT_SCALE_ISSUE) ? 2 + kCpWarps : -1;
