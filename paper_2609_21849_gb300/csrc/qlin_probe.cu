@@ -247,6 +247,161 @@ cudaError_t launch_probe(int ctas, int iters, unsigned long long* out, unsigned*
   return cudaLaunchKernelEx(&cfg, kern, iters, out, err);
 }
 
+// ------------------------------------------------- scale-copy issue rate ---
+// One CTA pair: thread 0 of CTA 0 issues `mmas` NVFP4 pair MMAs (N = 256) per
+// iteration while `warps` warps of CTA 0 (lane 0 each) issue `copies`
+// tcgen05.cp.cta_group::2.32x128b.warpx4 per iteration between them, into
+// TMEM columns away from the MMAs' (the accumulator and its scale columns).
+// Per pair: out[0] the MMA thread's cycles, out[1] the first copy warp's
+// cycles until all copies (every warp's) have completed.
+constexpr int kCpThreads = 320;               // warp 0 MMA, warp 1 TMEM, warps 2-9 copies
+constexpr int kCpSmem = 160 * 1024;
+constexpr int kCpSrc = 65536;                 // copy sources: 16 slots of 4 KB
+static_assert(1024 + kCpSrc + 16 * 4096 <= kCpSmem, "copy probe buffers");
+
+__global__ void __launch_bounds__(kCpThreads, 1)
+    cp_probe_kernel(int iters, int mmas, int copies, int warps, unsigned long long* out,
+                    unsigned* err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = base;
+  uint8_t* sB = base + kASmem;
+  uint8_t* sSF = base + 49152;
+  uint8_t* sCp = base + kCpSrc;
+  __shared__ uint64_t bar[3];
+  __shared__ uint32_t tmem_slot;
+  for (int i = threadIdx.x; i < (kCpSrc + 16 * 4096) / 4; i += kCpThreads) {
+    uint32_t v = hash32((uint32_t)i * 2654435761u + blockIdx.x);
+    // operands hashed; the scale region and the copy sources hold 1.0 (0x38)
+    reinterpret_cast<uint32_t*>(base)[i] = (i >= 49152 / 4) ? 0x38383838u : v;
+  }
+  const uint32_t rank = cluster_ctarank();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    mbar_init(&bar[2], warps);
+    mbar_fence_init();
+  }
+  if (warp == 1) tmem_alloc_pair(&tmem_slot, 512);
+  fence_proxy_async_smem();
+  tc_fence_before();
+  cluster_sync();
+  tc_fence_after();
+  const uint32_t tb = tmem_slot;
+  const uint32_t sf_t = tb + 256;   // the MMAs' scale columns (256..267)
+  if (threadIdx.x == 0 && rank == 0) {
+    for (int r = 0; r < 3; ++r) tc_cp_scales_pair(sf_t + 4 * r, sdesc_scales(smem_u32(sSF) + 512 * r));
+    tc_commit_pair_mc(&bar[0], 1);
+    (void)probe_wait(&bar[0], 0, err);
+  }
+  tc_fence_before();
+  cluster_sync();
+  tc_fence_after();
+  if (rank == 0 && warp == 0 && lane == 0) {
+    const uint32_t idesc = idesc_nvfp4(256, 256);
+    const uint32_t a = smem_u32(sA), b = smem_u32(sB);
+    const unsigned long long c0 = clock64();
+    for (int i = 0; i < iters; ++i)
+      for (int j = 0; j < mmas; ++j)
+        mma_nvfp4_pair(tb, sdesc_k128(a + (j & 3) * 32), sdesc_k128(b + (j & 3) * 32), idesc,
+                       sf_t, sf_t + 4, (i | j) ? 1u : 0u);
+    tc_commit_pair_mc(&bar[1], 1);
+    const bool ok = probe_wait(&bar[1], 0, err);
+    out[2 * (blockIdx.x / 2)] = ok ? clock64() - c0 : 0ull;
+  }
+  if (rank == 0 && lane == 0 && warp >= 2 && warp < 2 + warps) {
+    const int per = copies / warps;
+    const unsigned long long c0 = clock64();
+    for (int i = 0; i < iters; ++i)
+      for (int c = 0; c < per; ++c) {
+        const int k = (i * per + c + 5 * (warp - 2)) & 15;
+        tc_cp_scales_pair(tb + 320 + (uint32_t)((k & 7) * 8),
+                          sdesc_scales(smem_u32(sCp) + (uint32_t)k * 4096));
+      }
+    tc_commit_pair_mc(&bar[2], 1);
+    if (warp == 2) {
+      const bool ok = probe_wait(&bar[2], 0, err);
+      out[2 * (blockIdx.x / 2) + 1] = ok ? clock64() - c0 : 0ull;
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  cluster_sync();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tb, 512);
+  }
+}
+
+// ------------------------------------------- shared-memory fill rate ---
+// One CTA per SM: `threads` issuing threads (lane 0 of warps 0..threads-1)
+// each keep `depth` copies of 16 KB in flight into a ring of their own, for
+// `iters` copies: mode 0 tiled 2-D tensor copies (a 128-row x 128-byte box,
+// 128-byte swizzle, from a [rows, 1536-byte] view of src, as the GEMM's
+// operand boxes), mode 1 plain bulk copies of 16 contiguous KB.  Box
+// positions are pseudo-random over src.  out[cta] = the first thread's
+// cycles until its last copy landed.
+constexpr int kFillThreads = 256;
+constexpr int kFillSmem = 200 * 1024;
+constexpr int kFillBox = 16384;
+constexpr int kFillRowBytes = 1536;
+
+__global__ void __launch_bounds__(kFillThreads, 1)
+    fill_probe_kernel(const __grid_constant__ CUtensorMap tm, const uint8_t* src,
+                      unsigned long long src_bytes, int mode, int threads, int depth, int iters,
+                      int rows, unsigned long long* out, unsigned* err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  __shared__ uint64_t bar[8][8];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int w = 0; w < 8; ++w)
+      for (int d = 0; d < 8; ++d) mbar_init(&bar[w][d], 1);
+    mbar_fence_init();
+  }
+  __syncthreads();
+  if (lane == 0 && warp < threads) {
+    uint8_t* ring = base + warp * depth * kFillBox;
+    uint32_t ph[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    unsigned long long r = ((unsigned long long)blockIdx.x * 8 + warp) * 7919ull + 1ull;
+    const unsigned long long c0 = clock64();
+    int issued = 0;
+    bool ok = true;
+    for (int i = 0; i < iters; ++i) {
+      const int sl = i % depth;
+      if (i >= depth) {
+        if (!probe_wait(&bar[warp][sl], ph[sl], err)) {
+          ok = false;
+          break;
+        }
+        ph[sl] ^= 1u;
+      }
+      mbar_arrive_expect_tx(&bar[warp][sl], kFillBox);
+      r = r * 6364136223846793005ull + 1442695040888963407ull;
+      if (mode == 0) {
+        const int x = (int)((r >> 33) % (unsigned long long)(kFillRowBytes / 128)) * 128;
+        const int y = (int)((r >> 13) % (unsigned long long)(rows / 128)) * 128;
+        tma_load_2d(ring + sl * kFillBox, &tm, &bar[warp][sl], x, y);
+      } else {
+        const unsigned long long off = ((r >> 20) % (src_bytes / kFillBox)) * kFillBox;
+        bulk_load(ring + sl * kFillBox, src + off, kFillBox, &bar[warp][sl]);
+      }
+      ++issued;
+    }
+    // the copies still in flight land before the CTA exits
+    for (int k = 0; k < depth && k < issued; ++k) {
+      const int sl = (issued - 1 - k) % depth;
+      if (!probe_wait(&bar[warp][sl], ph[sl], err)) ok = false;
+      ph[sl] ^= 1u;
+    }
+    if (warp == 0) out[blockIdx.x] = ok ? clock64() - c0 : 0ull;
+  }
+  __syncthreads();
+}
+
 }  // namespace
 }  // namespace qlin
 
@@ -277,4 +432,69 @@ extern "C" int qlin_probe_mma(int kind, int pair, int n, int ctas, int iters,
 #undef QLIN_PROBE_CASE
   if (!matched) return 1;
   return e == cudaSuccess ? 0 : 4;
+}
+
+extern "C" int qlin_probe_scale_copy(int warps, int copies, int mmas, int ctas, int iters,
+                                     unsigned long long* out, unsigned* err, void* stream) {
+  if (out == nullptr || err == nullptr || iters < 1 || ctas < 2 || ctas % 2 != 0) return 1;
+  if (warps < 1 || warps > 8 || copies < 0 || copies % warps != 0 || mmas < 0 || mmas > 16)
+    return 1;
+  if (cudaFuncSetAttribute(cp_probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           kCpSmem) != cudaSuccess)
+    return 4;
+  cudaLaunchConfig_t cfg{};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3((unsigned)ctas, 1, 1);
+  cfg.blockDim = dim3(kCpThreads, 1, 1);
+  cfg.dynamicSmemBytes = kCpSmem;
+  cfg.stream = static_cast<cudaStream_t>(stream);
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, cp_probe_kernel, iters, mmas, copies, warps, out, err) ==
+                 cudaSuccess
+             ? 0
+             : 4;
+}
+
+extern "C" int qlin_probe_fill(int mode, int threads, int depth, int ctas, int iters,
+                               const void* src, unsigned long long src_bytes,
+                               unsigned long long* out, unsigned* err, void* stream) {
+  if (out == nullptr || err == nullptr || src == nullptr || iters < 1 || ctas < 1) return 1;
+  if ((mode != 0 && mode != 1) || threads < 1 || threads > 8 || depth < 1 || depth > 8 ||
+      1024 + threads * depth * kFillBox > kFillSmem)
+    return 1;
+  const unsigned long long rows = src_bytes / kFillRowBytes / 128 * 128;
+  if (rows < 128 || rows > (1ull << 30) || (reinterpret_cast<uintptr_t>(src) & 127u) != 0)
+    return 1;
+  using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                       &q) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess || fn == nullptr)
+    return 4;
+  CUtensorMap tm;
+  const cuuint64_t dims[2] = {(cuuint64_t)kFillRowBytes, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)kFillRowBytes};
+  const cuuint32_t box[2] = {128, 128};
+  const cuuint32_t es[2] = {1, 1};
+  if (reinterpret_cast<EncodeFn>(fn)(&tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(src),
+                                     dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return 1;
+  if (cudaFuncSetAttribute(fill_probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           kFillSmem) != cudaSuccess)
+    return 4;
+  fill_probe_kernel<<<ctas, kFillThreads, kFillSmem, static_cast<cudaStream_t>(stream)>>>(
+      tm, static_cast<const uint8_t*>(src), src_bytes, mode, threads, depth, iters, (int)rows,
+      out, err);
+  return cudaGetLastError() == cudaSuccess ? 0 : 4;
 }

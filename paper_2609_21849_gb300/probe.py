@@ -1,12 +1,17 @@
 """Tensor-core rate probe (include/qlin_probe.h): the measured ceiling of the
-tcgen05 MMA forms the GEMMs issue, for the roofline fractions.
+tcgen05 MMA forms the GEMMs issue, for the roofline fractions, and the issue
+rates of the copies that feed them.
 
-  python -m paper_2609_21849_gb300.probe
+  python -m paper_2609_21849_gb300.probe            # MMA ceilings
+  python -m paper_2609_21849_gb300.probe --copies   # block-scale copy and fill rates
 
-Each case runs back-to-back MMAs of one kind and shape from one thread per
+Each MMA case runs back-to-back MMAs of one kind and shape from one thread per
 CTA (or CTA pair) on every SM at once; the result is FLOP per SM cycle
 (clock-independent), the SM clock the probe ran at (cycles / nanoseconds)
-and the rate in TFLOP/s there and at the maximum SM clock.
+and the rate in TFLOP/s there and at the maximum SM clock.  The copy cases
+give SM cycles per stage's worth of block-scale copies against the number of
+issuing warps, and shared-memory fill bytes per cycle per SM against the
+number of threads issuing copies.
 """
 from __future__ import annotations
 
@@ -41,6 +46,11 @@ def _load():
         lib = ctypes.CDLL(build.PROBE_LIB)
         lib.qlin_probe_mma.restype = ctypes.c_int
         lib.qlin_probe_mma.argtypes = [ctypes.c_int] * 5 + [ctypes.c_void_p] * 3
+        lib.qlin_probe_scale_copy.restype = ctypes.c_int
+        lib.qlin_probe_scale_copy.argtypes = [ctypes.c_int] * 5 + [ctypes.c_void_p] * 3
+        lib.qlin_probe_fill.restype = ctypes.c_int
+        lib.qlin_probe_fill.argtypes = ([ctypes.c_int] * 5 + [ctypes.c_void_p, ctypes.c_ulonglong]
+                                        + [ctypes.c_void_p] * 3)
         _lib = lib
     return _lib
 
@@ -78,5 +88,66 @@ def ceilings(sm_max_mhz: float = 2070.0) -> dict:
             for (name, kind, pair, n, k) in CASES}
 
 
+def scale_copy_cycles(warps: int, copies: int = 12, mmas: int = 4, iters: int = 2000) -> dict:
+    """SM cycles per iteration of `mmas` NVFP4 pair MMAs (N = 256) and, beside
+    them, `copies` block-scale copies issued from `warps` warps (mmas = 0:
+    the copies alone), every SM pair at once."""
+    lib = _load()
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    ctas = sms // 2 * 2
+    out = torch.zeros(ctas, dtype=torch.int64, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    s = torch.cuda.current_stream().cuda_stream
+    for it in (64, iters):
+        st = lib.qlin_probe_scale_copy(warps, copies, mmas, ctas, it, out.data_ptr(), err.data_ptr(), s)
+        if st != 0:
+            raise RuntimeError(f"qlin_probe_scale_copy({warps}, {copies}, {mmas}) returned {st}")
+    torch.cuda.synchronize()
+    if int(err.item()) != 0:
+        raise RuntimeError("probe wait expired")
+    v = out.view(-1, 2).cpu().double()
+    mma = v[:, 0].median().item() / iters if mmas else None
+    cp = v[:, 1].median().item() / iters if copies else None
+    return {"warps": warps, "copies": copies, "mmas": mmas,
+            "mma_cycles_per_iter": None if mma is None else round(mma, 1),
+            "copy_cycles_per_iter": None if cp is None else round(cp, 1)}
+
+
+def fill_bytes_per_cycle(mode: int, threads: int, depth: int, iters: int = 3000,
+                         src_mb: int = 24) -> dict:
+    """Shared-memory fill rate per SM (bytes per SM cycle), every SM at once,
+    of `threads` threads each keeping `depth` 16 KB copies in flight: mode 0
+    tiled 128-byte-swizzled tensor boxes, mode 1 plain bulk copies; the
+    source (src_mb MB) stays in L2, as the GEMMs' operands do."""
+    lib = _load()
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    nbytes = (src_mb << 20) // (1536 * 128) * (1536 * 128)
+    src = torch.randint(0, 255, (nbytes,), dtype=torch.uint8, device="cuda")
+    out = torch.zeros(sms, dtype=torch.int64, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    s = torch.cuda.current_stream().cuda_stream
+    for it in (64, iters):
+        st = lib.qlin_probe_fill(mode, threads, depth, sms, it, src.data_ptr(), nbytes,
+                                 out.data_ptr(), err.data_ptr(), s)
+        if st != 0:
+            raise RuntimeError(f"qlin_probe_fill({mode}, {threads}, {depth}) returned {st}")
+    torch.cuda.synchronize()
+    if int(err.item()) != 0:
+        raise RuntimeError("probe wait expired")
+    cyc = out.cpu().double().median().item()
+    return {"mode": ("tiled_128B_box", "bulk")[mode], "threads": threads, "depth": depth,
+            "bytes_per_cycle_per_sm": round(threads * iters * 16384 / cyc, 1)}
+
+
+def copy_rates() -> dict:
+    cp = [scale_copy_cycles(w, 12, 0) for w in (1, 2, 4, 6)]
+    cp += [scale_copy_cycles(w, 12, 4) for w in (1, 2, 4, 6)]
+    cp += [scale_copy_cycles(1, 0, 4)]
+    fill = [fill_bytes_per_cycle(m, t, d) for m in (0, 1)
+            for (t, d) in ((1, 2), (1, 8), (2, 4), (4, 2), (6, 2), (8, 1))]
+    return {"scale_copy": cp, "fill": fill}
+
+
 if __name__ == "__main__":
-    print(json.dumps(ceilings(), indent=1))
+    import sys
+    print(json.dumps(copy_rates() if "--copies" in sys.argv[1:] else ceilings(), indent=1))

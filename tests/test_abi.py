@@ -41,17 +41,33 @@ def test_probe_library_exports_its_header(lib):
     from paper_2609_21849_gb300 import build
     probe = ctypes.CDLL(build.PROBE_LIB)
     names = _declared("qlin_probe.h")
-    assert names == ["qlin_probe_mma"]
+    assert names == ["qlin_probe_fill", "qlin_probe_mma", "qlin_probe_scale_copy"]
     for name in names:
         assert hasattr(probe, name), name
     f = probe.qlin_probe_mma
     f.restype = ctypes.c_int
     f.argtypes = [ctypes.c_int] * 5 + [ctypes.c_void_p] * 3
     one = ctypes.c_ulonglong(0)
+    p1 = ctypes.addressof(one)
     # argument errors are returned before any launch
-    assert f(4, 1, 256, 3, 16, ctypes.addressof(one), ctypes.addressof(one), None) == 1  # odd pair grid
-    assert f(4, 0, 64, 2, 16, ctypes.addressof(one), ctypes.addressof(one), None) == 1   # no such case
+    assert f(4, 1, 256, 3, 16, p1, p1, None) == 1  # odd pair grid
+    assert f(4, 0, 64, 2, 16, p1, p1, None) == 1   # no such case
     assert f(4, 0, 256, 2, 16, None, None, None) == 1
+    g = probe.qlin_probe_scale_copy
+    g.restype = ctypes.c_int
+    g.argtypes = [ctypes.c_int] * 5 + [ctypes.c_void_p] * 3
+    assert g(4, 12, 4, 3, 16, p1, p1, None) == 1   # odd pair grid
+    assert g(5, 12, 4, 2, 16, p1, p1, None) == 1   # copies not a multiple of the warps
+    assert g(9, 18, 4, 2, 16, p1, p1, None) == 1   # more than 8 copy warps
+    assert g(4, 12, 4, 2, 16, None, None, None) == 1
+    h = probe.qlin_probe_fill
+    h.restype = ctypes.c_int
+    h.argtypes = [ctypes.c_int] * 5 + [ctypes.c_void_p, ctypes.c_ulonglong] + [ctypes.c_void_p] * 3
+    big = 1 << 30   # never dereferenced: the checks fail first
+    assert h(2, 4, 2, 1, 16, 256, big, p1, p1, None) == 1          # no such mode
+    assert h(0, 8, 8, 1, 16, 256, big, p1, p1, None) == 1          # 1 MB of rings
+    assert h(0, 4, 2, 1, 16, 256, 1536 * 64, p1, p1, None) == 1    # fewer than 128 rows
+    assert h(0, 4, 2, 1, 16, 256 + 64, big, p1, p1, None) == 1     # source not 128-byte aligned
 
 
 def test_scale_bytes_and_workspace(lib):
