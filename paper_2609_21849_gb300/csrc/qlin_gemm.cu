@@ -141,6 +141,7 @@ struct KParams {
   float* y_sdec;            // with y_amax: where the last CTA writes S_dec = amax / 2688
   int fp16;           // 16-bit operand kernel only: fp16 operands and output (else bf16)
   int y_v8;           // y is 32-byte aligned: direct stores may use 32-byte vectors
+  int rq_v8;          // the re-quantized codes are 32-byte aligned: one 32-byte store per group
   unsigned* err;
   uint64_t timeout_ns;
 };
@@ -734,16 +735,24 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
             if (c64 < p.rq_col0 || c64 + 64 > p.rq_col0 + p.rq_cols || c64 >= p.N) continue;
             uint8_t* cp = p.rq_codes + row * p.rq_cols + (c64 - p.rq_col0);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {   // 16 columns per 16-byte store
-              const uint32_t* pk = packed + g * 32 + q * 8;
-              uint32_t w4[4];
+            for (int q2 = 0; q2 < 2; ++q2) {   // 32 columns per 32-byte store (or two 16-byte)
+              uint32_t w8[8];
 #pragma unroll
-              for (int i = 0; i < 4; ++i)
-                w4[i] = e4m3x4(__fmul_rn(bf16_lo(pk[2 * i]), s_enc_next),
-                               __fmul_rn(bf16_hi(pk[2 * i]), s_enc_next),
-                               __fmul_rn(bf16_lo(pk[2 * i + 1]), s_enc_next),
-                               __fmul_rn(bf16_hi(pk[2 * i + 1]), s_enc_next));
-              st_global_v4(cp + 16 * q, w4[0], w4[1], w4[2], w4[3]);
+              for (int h = 0; h < 2; ++h) {
+                const uint32_t* pk = packed + g * 32 + (2 * q2 + h) * 8;
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                  w8[4 * h + i] = e4m3x4(__fmul_rn(bf16_lo(pk[2 * i]), s_enc_next),
+                                         __fmul_rn(bf16_hi(pk[2 * i]), s_enc_next),
+                                         __fmul_rn(bf16_lo(pk[2 * i + 1]), s_enc_next),
+                                         __fmul_rn(bf16_hi(pk[2 * i + 1]), s_enc_next));
+              }
+              if (p.rq_v8) {
+                st_global_v8(cp + 32 * q2, w8);
+              } else {
+                st_global_v4(cp + 32 * q2, w8[0], w8[1], w8[2], w8[3]);
+                st_global_v4(cp + 32 * q2 + 16, w8[4], w8[5], w8[6], w8[7]);
+              }
             }
           }
         }
@@ -778,8 +787,14 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
               }
             }
             uint8_t* cp = p.rq_codes + row * (p.rq_cols / 2) + lc / 2;
-            st_global_v4(cp, words[0], words[1], words[2], words[3]);
-            st_global_v4(cp + 16, words[4], words[5], words[6], words[7]);
+            // the group's 32 bytes of codes: one store where aligned (each
+            // store instruction of the epilogue slows the mainloop beside it)
+            if (p.rq_v8) {
+              st_global_v8(cp, words);
+            } else {
+              st_global_v4(cp, words[0], words[1], words[2], words[3]);
+              st_global_v4(cp + 16, words[4], words[5], words[6], words[7]);
+            }
             *reinterpret_cast<uint32_t*>(p.rq_scales + scale_offset(row, lc / 16, p.rq_cols)) = sw;
           }
         }
@@ -946,6 +961,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, int num_sms, unsigned*
   p.y_sdec = a.y_sdec;
   p.fp16 = kBf16 && a.fp16 ? 1 : 0;
   p.y_v8 = (reinterpret_cast<uintptr_t>(a.y) & 31u) == 0 ? 1 : 0;
+  p.rq_v8 = (reinterpret_cast<uintptr_t>(a.rq_codes) & 31u) == 0 ? 1 : 0;
   p.err = err;
   p.timeout_ns = timeout_ns;
   auto kern = gemm_kernel<kFp4, kBN, kPair, kRequant, kBf16>;
