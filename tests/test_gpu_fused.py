@@ -95,7 +95,9 @@ def test_fused_qkv_value_window():
 @pytest.mark.parametrize("M,N,K,c0,cols", [(77, 320, 192, 64, 192), (1300, 3648, 320, 0, 3648),
                                            (513, 1024, 2560, 512, 512),
                                            # CTA pairs: partial last wave, row block and N block
-                                           (4500, 12224, 1024, 0, 12224)])
+                                           (4500, 12224, 1024, 0, 12224),
+                                           # CTA pairs with a partial last K stage (one MMA step)
+                                           (2048, 4096, 1088, 0, 4096)])
 def test_fused_ragged(M, N, K, c0, cols):
     x = synthetic.act_entry_outliers(M * 3 + K, M, K)
     (w,) = synthetic.weights(M * 3 + K, [(N, K)], 0.02)

@@ -65,7 +65,9 @@ def test_nvfp4_tiny_all_outputs():
 # ragged shapes: partial M and N tiles, K not a multiple of a pipeline stage,
 # both tile widths (128 x 128 when the 128 x 256 grid would not fill the GPU)
 RAGGED = [(1, 64, 64), (77, 320, 192), (300, 128, 512), (129, 576, 1088),
-          (1300, 3648, 320), (2048, 4096, 256)]
+          (1300, 3648, 320), (2048, 4096, 256),
+          # CTA pairs (256 x 256 tiles fill the GPU) with a partial last K stage
+          (2048, 4096, 1088)]
 
 
 @pytest.mark.parametrize("M,N,K", RAGGED)
