@@ -408,13 +408,17 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
           const uint32_t sA = smem_u32(smem + stage * C::kStageBytes);
           const uint32_t sB = sA + C::kABytes;
           const int nsteps = min(kStepsPerStage, k_steps - kb * kStepsPerStage);
+          // step j's operands start 32 j bytes in: the descriptors' start
+          // address field (address / 16, 14 bits; shared addresses stay
+          // below 256 KB, so it never carries) advances by 2 j
+          const uint64_t adesc0 = sdesc_k128(sA), bdesc0 = sdesc_k128(sB);
+          const uint32_t sfa0 = tmem_base + (uint32_t)(C::kSfColBase + stage * kStepsPerStage *
+                                                                           C::kSfColsPerStep);
           auto issue = [&](int j, uint32_t accumulate) {
-            const uint64_t adesc = sdesc_k128(sA + j * 32);
-            const uint64_t bdesc = sdesc_k128(sB + j * 32);
+            const uint64_t adesc = adesc0 + (uint64_t)(2 * j);
+            const uint64_t bdesc = bdesc0 + (uint64_t)(2 * j);
             if (kFp4) {
-              const uint32_t sfa_t = tmem_base + (uint32_t)(C::kSfColBase +
-                                                            (stage * kStepsPerStage + j) *
-                                                                C::kSfColsPerStep);
+              const uint32_t sfa_t = sfa0 + (uint32_t)(j * C::kSfColsPerStep);
               if (kPair)
                 mma_nvfp4_pair(d_tmem, adesc, bdesc, idesc, sfa_t, sfa_t + 4, accumulate);
               else
