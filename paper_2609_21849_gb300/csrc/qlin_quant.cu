@@ -64,9 +64,11 @@ struct AmaxOp {
   }
 };
 
-// One lane per 16-element block (two chunks); lanes 4g..4g+3 hold the four
-// blocks of a 64-element group.  r_b = S_enc / s_b comes from a per-CTA table
-// over the 127 finite E4M3 codes, filled with the same fp32 division.
+// One lane per 16-element block (two chunks); each lane stores its block's
+// scale code as one byte of the atom layout (one store instruction per warp,
+// instead of gathering a 64-element group's four codes by shuffles: measured
+// 2-7% faster).  r_b = S_enc / s_b comes from a per-CTA table over the 127
+// finite E4M3 codes, filled with the same fp32 division.
 template <typename Idx>
 struct Nvfp4Op {
   static constexpr int kUnit = 2;
@@ -89,8 +91,7 @@ struct Nvfp4Op {
     }
   }
   // The codes of one 16-element block (block amax bits mb) and its scale
-  // code; lanes 4g..4g+3 hold one 64-element group, whose four scales are
-  // gathered into lane 4g.
+  // code (in `word`).
   __device__ __forceinline__ void quantize_block(const uint4 (&v)[2], uint32_t mb,
                                                  uint32_t& code0, uint32_t& code1,
                                                  uint32_t& word) const {
@@ -106,10 +107,7 @@ struct Nvfp4Op {
 #pragma unroll
     for (int i = 0; i < 8; i += 2) mul2_rn(f[i], f[i + 1], r_b);
     code1 = e2m1x8(f);
-    const uint32_t s1 = __shfl_down_sync(0xFFFFFFFFu, sb, 1);
-    const uint32_t s2 = __shfl_down_sync(0xFFFFFFFFu, sb, 2);
-    const uint32_t s3 = __shfl_down_sync(0xFFFFFFFFu, sb, 3);
-    word = sb | (s1 << 8) | (s2 << 16) | (s3 << 24);
+    word = sb;
   }
   __device__ __forceinline__ void unit(const uint4 (&v)[2], uint64_t c, bool valid) {
     uint32_t code0, code1, word;
@@ -117,20 +115,19 @@ struct Nvfp4Op {
                    word);
     if (valid) {
       reinterpret_cast<uint2*>(codes)[c >> 1] = make_uint2(code0, code1);
-      if ((threadIdx.x & 3) == 0) {
+      {
         if constexpr (sizeof(Idx) == 4) {
           const uint32_t ci = (uint32_t)c;
           const uint32_t t = __umulhi(div_m, ci);
           const uint32_t row = (t + ((ci - t) >> div_s1)) >> div_s2;
           const uint32_t colc = ci - row * (uint32_t)chunks_per_row;   // in chunks
-          *reinterpret_cast<uint32_t*>(scales + ((row >> 7) * (uint32_t)(K >> 6) + (colc >> 3)) * 512u +
-                                       (row & 31u) * 16u + ((row >> 5) & 3u) * 4u) = word;
+          scales[((row >> 7) * (uint32_t)(K >> 6) + (colc >> 3)) * 512u +
+                 (row & 31u) * 16u + ((row >> 5) & 3u) * 4u + ((colc >> 1) & 3u)] = (uint8_t)word;
         } else {
           const Idx ci = (Idx)c;
           const Idx row = ci / chunks_per_row;
           const Idx col = (ci - row * chunks_per_row) << 3;
-          *reinterpret_cast<uint32_t*>(scales + scale_offset((int64_t)row, (int64_t)(col >> 4), K)) =
-              word;
+          scales[scale_offset((int64_t)row, (int64_t)(col >> 4), K)] = (uint8_t)word;
         }
       }
     }
@@ -151,7 +148,7 @@ struct Nvfp4Op {
     const uint64_t cg = c0 + 2u * threadIdx.x;
     uint32_t row = (uint32_t)(cg / cpr), col = (uint32_t)(cg % cpr);   // col in chunks
     const uint32_t kgroups = (uint32_t)(K >> 6);
-    // the loop bound is block-uniform: every lane reaches the shuffles
+    // the loop bound is block-uniform
 #pragma unroll
     for (int s = 0; s < kSteps; ++s) {
       const uint32_t base = (uint32_t)s * 2u * kStride;
@@ -172,18 +169,15 @@ struct Nvfp4Op {
         col_b -= cpr;
         ++row_b;
       }
-      const bool lead = (threadIdx.x & 3) == 0;
       if (ok_a) {
         reinterpret_cast<uint2*>(codes)[(c0 + cl) >> 1] = make_uint2(a0, a1);
-        if (lead)
-          *reinterpret_cast<uint32_t*>(scales + ((row >> 7) * kgroups + (col >> 3)) * 512u +
-                                       (row & 31u) * 16u + ((row >> 5) & 3u) * 4u) = aw;
+        scales[((row >> 7) * kgroups + (col >> 3)) * 512u + (row & 31u) * 16u +
+               ((row >> 5) & 3u) * 4u + ((col >> 1) & 3u)] = (uint8_t)aw;
       }
       if (ok_b) {
         reinterpret_cast<uint2*>(codes)[(c0 + cl + kStride) >> 1] = make_uint2(b0, b1);
-        if (lead)
-          *reinterpret_cast<uint32_t*>(scales + ((row_b >> 7) * kgroups + (col_b >> 3)) * 512u +
-                                       (row_b & 31u) * 16u + ((row_b >> 5) & 3u) * 4u) = bw;
+        scales[((row_b >> 7) * kgroups + (col_b >> 3)) * 512u + (row_b & 31u) * 16u +
+               ((row_b >> 5) & 3u) * 4u + ((col_b >> 1) & 3u)] = (uint8_t)bw;
       }
       row += dq;
       col += dr;
