@@ -577,10 +577,19 @@ __global__ void __launch_bounds__(Cfg<kFp4, kBN, kPair>::kThreads, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int ct = cid; ct < num_ctiles; ct += ncl) {
-      if (!mbar_wait(&tmem_full[acc], acc_phase, ctl)) break;
-      tc_fence_after();
       int mg, nb;
       tile_coords(ct, groups_m, tiles_n, &mg, &nb);
+      if (!kFp4 && !kBf16 && p.w_per_channel) {
+        // FP8: this tile's per-channel weight scales into L1 while the
+        // accumulator is still being computed (lane i: the 128-byte line of
+        // chunk i), so that the epilogue's loads of them wait on L1 rather
+        // than L2 -- the last tile's epilogue is on the kernel's critical path
+        const int64_t cl = (int64_t)nb * kBN + half * kCols + 32 * lane;
+        if (lane < kCols / 32 && cl < p.N)
+          asm volatile("prefetch.global.L1 [%0];" ::"l"(p.sdec_w + cl));
+      }
+      if (!mbar_wait(&tmem_full[acc], acc_phase, ctl)) break;
+      tc_fence_after();
       const int mb = mg * kCM + rank;
       const int64_t row = (int64_t)mb * kBM + quarter * 32 + lane;
       // chunk c (32 columns) of this thread starts at column ccol(c)
