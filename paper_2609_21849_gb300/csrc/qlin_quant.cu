@@ -310,11 +310,31 @@ __device__ __forceinline__ bool stream_tiles(const uint4* __restrict__ x, uint64
   return ok;
 }
 
+// The CTA's first kStages tiles (the ones stream_tiles copies first) into
+// L2, one bulk prefetch per tile from threads 0..kStages-1.  Called before
+// grid_dep_wait: a prefetch is a hint that returns no data, so it is correct
+// even while the previous kernel still writes x, and it lets the first
+// tiles' DRAM reads overlap that kernel's tail (NVFP4 4608 x 3072 static:
+// 9.17 -> 7.93 us in a chain of launches).
+__device__ __forceinline__ void l2_prefetch_first_tiles(const uint4* x, uint64_t n_chunks) {
+  const uint64_t n_tiles = (n_chunks + kTileChunks - 1) / kTileChunks;
+  if (threadIdx.x < kStages) {
+    const uint64_t t = blockIdx.x + (uint64_t)threadIdx.x * gridDim.x;
+    if (t < n_tiles) {
+      const uint64_t c0 = t * kTileChunks;
+      const uint64_t left = n_chunks - c0;
+      const uint32_t nc = left < (uint64_t)kTileChunks ? (uint32_t)left : (uint32_t)kTileChunks;
+      l2_prefetch_bulk(x + c0, nc * 16u);
+    }
+  }
+}
+
 // amax over n_chunks 16-byte chunks, folded into *amax_bits (fp32 bits;
 // cleared before the launch).
 __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
     amax_kernel(const uint4* __restrict__ x, uint64_t n_chunks, unsigned* __restrict__ amax_bits,
                 unsigned* err, uint64_t timeout_ns) {
+  l2_prefetch_first_tiles(x, n_chunks);
   grid_dep_wait();
   grid_dep_launch();
   __shared__ uint32_t warp_max[kThreads / 32];
@@ -353,6 +373,7 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
                        const float* scale_src, float* sdec_out, uint32_t* __restrict__ codes,
                        uint8_t* __restrict__ scales, uint3 row_div, unsigned* err,
                        uint64_t timeout_ns) {
+  l2_prefetch_first_tiles(x, n_chunks);
   grid_dep_wait();
   grid_dep_launch();
   __shared__ float r_table[128];
@@ -378,6 +399,7 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
     quant_fp8_kernel(const uint4* __restrict__ x, uint64_t n_chunks, const float* scale_src,
                      float* sdec_out, uint2* __restrict__ codes, unsigned* err,
                      uint64_t timeout_ns) {
+  l2_prefetch_first_tiles(x, n_chunks);
   grid_dep_wait();
   grid_dep_launch();
   Fp8Op op;
