@@ -221,8 +221,11 @@ struct Fp8Op {
 // flight; every thread applies `op` to its chunks of each landed tile.
 // `setup(op)` runs once the first copies are on their way (reads that only
 // the arithmetic needs, such as the tensor scale, overlap the loads).
-// Returns false if a bounded wait expired (recorded in *err).
-template <typename Op, typename Setup>
+// kReverse visits the tiles last-first: a second pass over data that a
+// first pass has just streamed forward starts on the lines still in L2
+// (NVFP4 dynamic route at 18432 x 3072, amax pass then quantizer: 49.5 ->
+// 48.2 us).  Returns false if a bounded wait expired (recorded in *err).
+template <bool kReverse = false, typename Op, typename Setup>
 __device__ __forceinline__ bool stream_tiles(const uint4* __restrict__ x, uint64_t n_chunks,
                                              Op& op, Setup setup, unsigned* err,
                                              uint64_t timeout_ns) {
@@ -234,7 +237,7 @@ __device__ __forceinline__ bool stream_tiles(const uint4* __restrict__ x, uint64
   const int tid = threadIdx.x;
 
   auto issue = [&](uint64_t t, int s) {
-    const uint64_t c0 = t * kTileChunks;
+    const uint64_t c0 = (kReverse ? n_tiles - 1 - t : t) * kTileChunks;
     const uint64_t left = n_chunks - c0;
     const uint32_t nc = left < (uint64_t)kTileChunks ? (uint32_t)left : (uint32_t)kTileChunks;
     mbar_arrive_expect_tx(&full[s], nc * 16u);
@@ -268,7 +271,7 @@ __device__ __forceinline__ bool stream_tiles(const uint4* __restrict__ x, uint64
       t_stop = t;
       break;
     }
-    const uint64_t c0 = t * kTileChunks;
+    const uint64_t c0 = (kReverse ? n_tiles - 1 - t : t) * kTileChunks;
     constexpr int kU = Op::kUnit;
 #pragma unroll
     for (int u = 0; u < kTileChunks / (kU * kThreads); ++u) {
@@ -370,7 +373,10 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
                        const float* scale_src, float* sdec_out, uint32_t* __restrict__ codes,
                        uint8_t* __restrict__ scales, uint3 row_div, unsigned* err,
                        uint64_t timeout_ns) {
-  l2_prefetch_first_tile(x, n_chunks);
+  // The dynamic-scale instance is the second pass over x (after amax_kernel,
+  // or over y after the GEMM that reduced its amax): it reads last-first, and
+  // its first tiles are then the ones most recently in L2.
+  if (!kDynamic) l2_prefetch_first_tile(x, n_chunks);
   grid_dep_wait();
   grid_dep_launch();
   __shared__ float r_table[128];
@@ -383,7 +389,7 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm)
   op.K = K;
   op.codes = codes;
   op.scales = scales;
-  stream_tiles(
+  stream_tiles<kDynamic>(
       x, n_chunks, op,
       [&](Nvfp4Op<Idx>& o) {
         o.s_enc = encode_scale(tensor_scale<kDynamic>(scale_src, sdec_out, 2688.0f));
