@@ -470,6 +470,18 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
 }
 
+// Wait until at most `pending` (0-3) of this thread's cp.async groups are
+// still in flight (the operand must be an immediate; a constant argument
+// folds the switch).
+__device__ __forceinline__ void cp_async_wait_pending(int pending) {
+  switch (pending) {
+    case 3: asm volatile("cp.async.wait_group 3;" ::: "memory"); break;
+    case 2: asm volatile("cp.async.wait_group 2;" ::: "memory"); break;
+    case 1: asm volatile("cp.async.wait_group 1;" ::: "memory"); break;
+    default: asm volatile("cp.async.wait_group 0;" ::: "memory"); break;
+  }
+}
+
 // sync[0]: amax bits (fp32), sync[1]: arrival count, sync[2]: departure
 // count; all zero at launch, and the last CTA to depart zeroes them again, so
 // back-to-back launches (graph replays included) need no clearing between.
@@ -492,7 +504,10 @@ __global__ void __launch_bounds__(kOnePassThreads, 1)
   // every thread copies its chunks (a dozen 16-byte asynchronous copies in
   // flight per thread), then takes their amax; it reads only the chunks it
   // copied itself, so waiting for its own copies suffices.  NVFP4 copies in
-  // the units run_slice quantizes (two adjacent chunks, a warp covering 1 KB)
+  // the units run_slice quantizes (two adjacent chunks, a warp covering 1 KB),
+  // one copy group per step of block maxima, so that each step's maxima are
+  // taken while the later steps' copies are still landing (4608 x 3072:
+  // 12.46 -> 12.23 us)
   const uint4* xs = x + c_begin;
   if constexpr (Op::kBlockMax) {
 #pragma unroll
@@ -502,19 +517,23 @@ __global__ void __launch_bounds__(kOnePassThreads, 1)
         cp_async16(smem_u32(buf + c), xs + c);
         cp_async16(smem_u32(buf + c + 1), xs + c + 1);
       }
+      if (s & 1) asm volatile("cp.async.commit_group;" ::: "memory");   // step s / 2
     }
   } else {
     for (uint32_t i = tid; i < n; i += kOnePassThreads) cp_async16(smem_u32(buf + i), xs + i);
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
+    grid_dep_launch();   // x is on chip: the next kernel may begin launching
   }
-  asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
-  grid_dep_launch();   // x is on chip: the next kernel may begin launching
   uint32_t m = 0;
   uint32_t bm[kOnePassSteps] = {};
   if constexpr (Op::kBlockMax) {
     // NVFP4: the amax of each 16-element block this thread will quantize
     // (the units of run_slice), kept for after the barrier
+    static_assert(kOnePassSteps <= 4, "cp_async_wait_pending takes 0-3 groups");
 #pragma unroll
     for (int s = 0; s < kOnePassSteps; ++s) {
+      cp_async_wait_pending(kOnePassSteps - 1 - s);   // steps 0..s have landed
+      if (s == kOnePassSteps - 1) grid_dep_launch();  // x is on chip
       const uint32_t ca = (uint32_t)s * 4u * kOnePassThreads + 2u * tid;
       const uint32_t cb = ca + 2u * kOnePassThreads;
       const uint32_t a =
