@@ -147,6 +147,19 @@ def test_dynamic_scale_x_larger_than_on_chip(fmt):
         assert np.array_equal(u8(q.codes), rc)
 
 
+def test_dynamic_scale_two_pass_ragged_last_tile():
+    # 9217 x 4096 takes the amax pass + quantizer route and ends in a partial
+    # 16 KB tile (4 719 104 chunks of 16 bytes); the quantizer pass visits
+    # its tiles last-first, so that partial tile is the first it copies.
+    # Rows past the last 128-row atom are a ragged scale block as well.
+    M, K = 9217, 4096
+    assert (M * K // 8) % 1024 != 0
+    x = synthetic.act_entry_outliers(78, M, K)
+    q = qlin.qlin_quantize_act_nvfp4(to_dev(x))
+    assert qlin.qlin_sync_status() == 0
+    assert_nvfp4_equal(q, oracle.quant_nvfp4(x), "9217x4096 dynamic")
+
+
 def test_dynamic_scale_one_read_repeated():
     # the one-read route keeps its grid-wide amax in two scratch words that
     # each launch clears: back-to-back calls on tensors of decreasing amax
